@@ -1,0 +1,409 @@
+"""Pins of the CPU oracle to facts fixed by the paper and by mathematics.
+
+Each test checks the oracle against something other than itself: the paper's
+worked examples (golden fixtures), Theorem 1, the slack identity, the bounds
+of Propositions 1-3 with their tightness constructions, special cases that
+reduce to a library routine (numpy sort / median / argmax, Python sorted),
+brute-force single-rank-stall constructions, and hand-derived label fixtures.
+"""
+import itertools
+
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from tests.golden import fixtures
+
+LIMIT47 = 1 << 47
+
+
+def rand_d(rng, T, R, S, hi=10**6, zero_frac=0.0):
+    d = rng.integers(0, hi, size=(T, R, S), dtype=np.int64)
+    if zero_frac:
+        d[rng.random((T, R, S)) < zero_frac] = 0
+    return d
+
+
+# ---------------------------------------------------------------- worked examples
+
+def test_fig1_motivating_example():
+    g = fixtures.load("fig1_motivating.txt")
+    f = O.frontier(g["d"])
+    u = g["unit_ns"]
+    assert (f.a[0] == g["a"] * u).all()
+    assert f.makespan[0] == g["makespan"][0] * u
+    assert (f.lead[0] == g["lead"]).all()       # tie at bwd goes to the lowest rank, r0
+    assert (f.ties[0] == g["ties"]).all()
+    # the per-stage maximum the paper contrasts with the frontier
+    assert g["d"][0].max(axis=0).sum() == g["per_stage_max_total"][0] * u
+
+
+def test_fig2_frontier_example():
+    g = fixtures.load("fig2_frontier.txt")
+    f = O.frontier(g["d"])
+    u = g["unit_ns"]
+    assert (f.F[0] == g["F"] * u).all()
+    assert (f.a[0] == g["a"] * u).all()
+    assert f.makespan[0] == g["makespan"][0] * u
+    assert (f.lead[0] == g["lead"]).all()
+
+
+def test_sharp_cocritical_example():
+    g = fixtures.load("sharp_cocritical.txt")
+    W = int(g["W"][0])
+    d = np.repeat(g["d"], W, axis=0)
+    f = O.frontier(d)
+    u = g["unit_ns"]
+    assert (f.F == g["F"] * u).all() and (f.a == g["a"] * u).all() and (f.lead == g["lead"]).all()
+    L = O.label_windows(d, W)
+    assert L.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_CO_CRITICAL
+    assert L.amb_mask[0] == sum(1 << s for s in g["amb"])
+    assert L.route_mask[0] == 0b01
+    assert (L.Y == 0).all()
+
+
+# ---------------------------------------------------------------- Theorem 1 / identities
+
+@pytest.mark.parametrize("T,R,S", [(50, 1, 1), (40, 3, 5), (30, 17, 8), (10, 64, 13)])
+def test_telescoping_exact(T, R, S):
+    rng = np.random.default_rng(T * 1000 + R * 10 + S)
+    d = rand_d(rng, T, R, S, zero_frac=0.2)
+    f = O.frontier(d)
+    assert (f.a >= 0).all()
+    assert (f.a.sum(axis=1) == f.makespan).all()          # Theorem 1, exact in int64
+    assert (f.makespan == d.sum(axis=2).max(axis=1)).all()  # F_{t,S} is the largest rank total
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_slack_identity(seed):
+    rng = np.random.default_rng(seed)
+    T, R, S = 25, 7, 6
+    d = rand_d(rng, T, R, S, zero_frac=0.3)
+    f = O.frontier(d)
+    P = np.cumsum(d, axis=2)
+    Fprev = np.concatenate([np.zeros((T, 1), np.int64), f.F[:, :-1]], axis=1)
+    Pprev = np.concatenate([np.zeros((T, R, 1), np.int64), P[:, :, :-1]], axis=2)
+    lam = Fprev[:, None, :] - Pprev            # slack lambda_{t,r,s} >= 0
+    assert (lam >= 0).all()
+    assert (f.a == (d - lam).max(axis=1)).all()
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_prop1_prop2_bounds(seed):
+    rng = np.random.default_rng(100 + seed)
+    T, R, S = 40, 9, 5
+    d = rand_d(rng, T, R, S, zero_frac=0.3)
+    f = O.frontier(d)
+    M = d.max(axis=1).sum(axis=1)
+    Mbar_R = d.sum(axis=1).sum(axis=1)          # R * average summary, kept integral
+    F = f.makespan
+    assert (F <= M).all() and (M <= min(R, S) * F).all()
+    assert (F <= Mbar_R).all() and (Mbar_R <= R * F).all()
+
+
+@pytest.mark.parametrize("R,S", [(3, 5), (5, 3), (4, 4)])
+def test_prop1_tightness(R, S):
+    # min(R,S) distinct rank-stage pairs of duration D, no rank holding two
+    Dv = 7_000_000
+    d = np.zeros((1, R, S), np.int64)
+    for i in range(min(R, S)):
+        d[0, i, i] = Dv
+    f = O.frontier(d)
+    M = d.max(axis=1).sum()
+    assert M == min(R, S) * f.makespan[0]
+
+
+def test_prop2_tightness():
+    R, S = 6, 4
+    d = np.zeros((1, R, S), np.int64)
+    d[0, 2] = [1, 2, 3, 4]                      # one rank with total D, all others zero
+    f = O.frontier(d)
+    assert d.sum() == f.makespan[0]             # R * Mbar == F, i.e. Mbar = F / R
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_prop3_stability(seed):
+    rng = np.random.default_rng(200 + seed)
+    T, R, S, eps = 30, 6, 7, 1000
+    d = rand_d(rng, T, R, S, hi=10**6) + eps
+    delta = rng.integers(-eps, eps + 1, size=d.shape)
+    f0, f1 = O.frontier(d), O.frontier(d + delta)
+    s1 = np.arange(1, S + 1)                    # 1-based stage index
+    assert (np.abs(f1.F - f0.F) <= s1 * eps).all()
+    assert (np.abs(f1.a - f0.a) <= (2 * s1 - 1) * eps).all()
+
+
+# ---------------------------------------------------------------- special cases
+
+def test_single_rank_reduces_to_its_vector():
+    rng = np.random.default_rng(7)
+    d = rand_d(rng, 20, 1, 9)
+    f = O.frontier(d)
+    assert (f.a == d[:, 0, :]).all() and (f.lead == 0).all() and (f.ties == 1).all()
+
+
+def test_identical_ranks():
+    rng = np.random.default_rng(8)
+    base = rand_d(rng, 15, 1, 6)
+    d = np.repeat(base, 11, axis=1)
+    f = O.frontier(d)
+    assert (f.a == base[:, 0, :]).all() and (f.lead == 0).all() and (f.ties == 11).all()
+
+
+@pytest.mark.parametrize("R,S", [(2, 2), (3, 4), (5, 6)])
+def test_single_rank_stall_brute_force(R, S):
+    """Identical ranks, no sync stage, a stall Delta on (r*, s*): only a[s*]
+    grows, by exactly Delta, and r* leads every boundary from s* on."""
+    rng = np.random.default_rng(R * 10 + S)
+    base = rng.integers(1, 10**6, size=S, dtype=np.int64)
+    for r_star, s_star in itertools.product(range(R), range(S)):
+        Delta = int(rng.integers(1, 10**6))
+        d = np.tile(base, (1, R, 1))
+        d[0, r_star, s_star] += Delta
+        f = O.frontier(d)
+        exp_a = base.copy()
+        exp_a[s_star] += Delta
+        assert (f.a[0] == exp_a).all()
+        exp_lead = np.where(np.arange(S) >= s_star, r_star, 0)
+        assert (f.lead[0] == exp_lead).all()
+
+
+def test_rank_permutation_invariance():
+    rng = np.random.default_rng(9)
+    d = rand_d(rng, 12, 6, 5, hi=50)           # small values: many ties
+    perm = rng.permutation(6)
+    f0, f1 = O.frontier(d), O.frontier(d[:, perm, :])
+    assert (f0.F == f1.F).all() and (f0.a == f1.a).all() and (f0.ties == f1.ties).all()
+
+
+def test_input_errors():
+    d = np.ones((2, 3, 4), np.int64)
+    d[1, 2, 3] = -1
+    with pytest.raises(O.OracleError) as e:
+        O.frontier(d)
+    assert e.value.rc == O.NEGATIVE
+    d[1, 2, 3] = LIMIT47
+    with pytest.raises(O.OracleError) as e:
+        O.frontier(d)
+    assert e.value.rc == O.RANGE
+    d[1, 2, 3] = LIMIT47 // 2
+    d[1, 2, 2] = LIMIT47 // 2                   # prefix reaches 2^47
+    with pytest.raises(O.OracleError) as e:
+        O.frontier(d)
+    assert e.value.rc == O.RANGE
+
+
+# ---------------------------------------------------------------- windows (Eq. 2)
+
+@pytest.mark.parametrize("t0,W", [(0, 7), (5, 7), (13, 4), (0, 100)])
+def test_window_invariants(t0, W):
+    rng = np.random.default_rng(t0 + W)
+    T, R, S = 37, 5, 4
+    d = rand_d(rng, T, R, S, hi=30, zero_frac=0.2)   # many ties
+    w = O.windows(d, W, t0)
+    f = O.frontier(d)
+    nW = O.num_windows(t0, T, W)
+    assert w.X.shape == (nW, S)
+    assert (w.X.sum(axis=1) == w.D).all()
+    assert (w.E.sum(axis=2) == w.X).all()
+    g = np.arange(T) + t0
+    widx = g // W - t0 // W
+    n_w = np.bincount(widx, minlength=nW)
+    assert (w.C.sum(axis=2) == n_w[:, None]).all()
+    assert (w.step_lead == np.argmax(f.a, axis=1)).all()   # numpy argmax: first maximum
+    for i in range(nW):
+        sel = widx == i
+        assert (w.X[i] == f.a[sel].sum(axis=0)).all() and w.D[i] == f.makespan[sel].sum()
+
+
+def test_window_chunk_additivity():
+    rng = np.random.default_rng(11)
+    T, R, S, W = 60, 4, 3, 25
+    d = rand_d(rng, T, R, S)
+    whole = O.windows(d, W, 0)
+    a = O.windows(d[:35], W, 0)      # windows 0..1
+    b = O.windows(d[35:], W, 35)     # windows 1..2
+    X = np.zeros_like(whole.X)
+    X[:2] += a.X
+    X[1:] += b.X
+    assert (X == whole.X).all()
+
+
+# ---------------------------------------------------------------- top-k
+
+@pytest.mark.parametrize("seed", range(3))
+def test_topk_against_sorted(seed):
+    rng = np.random.default_rng(300 + seed)
+    nW, S, R, k = 3, 5, 7, 6
+    X = rng.integers(0, 4, size=(nW, S)).astype(np.int64)
+    E = rng.integers(0, 4, size=(nW, S, R)).astype(np.int64)
+    t = O.topk(X, E, k)
+    for w in range(nW):
+        st = sorted([(-X[w, s], s) for s in range(S) if X[w, s] > 0])[:k]
+        exp = [s for _, s in st] + [-1] * (k - len(st))
+        assert list(t.stage[w]) == exp
+        pr = sorted([(-E[w, s, r], s, r) for s in range(S) for r in range(R) if E[w, s, r] > 0])[:k]
+        exp_p = [[s, r] for _, s, r in pr] + [[-1, -1]] * (k - len(pr))
+        assert t.pair[w].tolist() == exp_p
+        assert list(t.pair_value[w]) == [-v for v, _, _ in pr] + [0] * (k - len(pr))
+
+
+# ---------------------------------------------------------------- median and gain (Eq. 3)
+
+@pytest.mark.parametrize("T,W", [(30, 10), (31, 10), (9, 4), (5, 16)])
+def test_median_is_lower_median(T, W):
+    rng = np.random.default_rng(T + W)
+    R, S = 3, 4
+    d = rand_d(rng, T, R, S, hi=20)
+    m = O.window_median(d, W)
+    for w in range((T + W - 1) // W):
+        blk = d[w * W:(w + 1) * W]
+        n = blk.shape[0]
+        assert (m[w] == np.sort(blk, axis=0)[(n - 1) // 2]).all()
+        if n % 2 == 1:
+            assert (m[w] == np.median(blk, axis=0)).all()
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_gain_closed_form_and_sign(seed):
+    """Replacing one stage shifts only the prefixes at and after it, so
+    F'_S = max_r (P_{t,r,S} - max(0, d_{t,r,s} - m_{r,s})); G_s >= 0."""
+    rng = np.random.default_rng(400 + seed)
+    T, R, S, W = 23, 6, 5, 8
+    d = rand_d(rng, T, R, S, hi=1000, zero_frac=0.1)
+    m = O.window_median(d, W)
+    Y = O.direct_gain(d, W, m)
+    assert (Y >= 0).all()
+    PS = d.sum(axis=2)
+    FS = PS.max(axis=1)
+    exp = np.zeros_like(Y)
+    for t in range(T):
+        w = t // W
+        cut = np.maximum(0, d[t] - m[w])            # [R][S]
+        Fp = (PS[t][:, None] - cut).max(axis=0)     # [S]
+        exp[w] += FS[t] - Fp
+    assert (Y == exp).all()
+
+
+def test_gain_single_rank_and_constant_window():
+    rng = np.random.default_rng(5)
+    d = rand_d(rng, 20, 1, 4)
+    W = 10
+    m = O.window_median(d, W)
+    Y = O.direct_gain(d, W, m)
+    for w in range(2):
+        assert (Y[w] == np.maximum(0, d[w * W:(w + 1) * W, 0, :] - m[w, 0]).sum(axis=0)).all()
+    const = np.repeat(rand_d(rng, 1, 5, 4), 12, axis=0)
+    assert (O.direct_gain(const, 6, O.window_median(const, 6)) == 0).all()
+
+
+# ---------------------------------------------------------------- labels: hand-derived fixtures
+
+U = 1_000_000  # 1 ms
+
+
+def _intermittent_data_stall():
+    """R=4, S=3, W=10, every duration 10 ms; r0's data +30 ms on steps 0-3.
+    Stalled steps: a=(40,10,10), F_S=60; others a=(10,10,10), F_S=30.
+    X=(220,100,100), D=420 -> A_data=0.524>0.4.  r0's data median over
+    {40 x4, 10 x6} is 10, so the clipped replacement removes the stall:
+    Y_data=4*(60-30)=120, G=0.286>=0.1 -> direct_exposure.  C_A=C_G={data}.
+    Only the 4 stalled steps are confident (margin 30 >= 0.05*60), all data."""
+    d = np.full((10, 4, 3), 10 * U, np.int64)
+    d[0:4, 0, 0] += 30 * U
+    return d
+
+
+def test_label_direct_exposure():
+    L = O.label_windows(_intermittent_data_stall(), 10)
+    assert (L.X[0] == np.array([220, 100, 100]) * U).all() and L.D[0] == 420 * U
+    assert (L.Y[0] == np.array([120, 0, 0]) * U).all()
+    assert L.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_DIRECT_EXPOSURE
+    assert L.amb_mask[0] == 0b001
+    # cumulative X: 220 < 336, 320 < 336, 420 >= 336 = 0.8*420
+    assert L.route_mask[0] == 0b111
+    assert L.n_confident[0] == 4 and L.n_switch[0] == 0
+    assert L.share[0, 0] == 220 / 420 and L.gain[0, 0] == 120 / 420
+
+
+def test_label_sync_wait_dependent_with_model_fit():
+    g = fixtures.load("sharp_cocritical.txt")
+    d = np.repeat(g["d"], 20, axis=0)
+    cfg = O.default_config()
+    cfg.model_fit_mask = 0b01                       # W_data = 1
+    L = O.label_windows(d, 20, cfg=cfg)
+    assert L.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_SYNC_WAIT_DEPENDENT
+    assert L.amb_mask[0] == 0b11
+
+
+def test_label_telemetry_limited_missing_rank():
+    L = O.label_windows(_intermittent_data_stall(), 10, missing=np.array([1]))
+    assert L.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_TELEMETRY_LIMITED
+
+
+def test_label_telemetry_limited_closure_and_overlap():
+    d = _intermittent_data_stall()
+    tot = d.sum(axis=2)
+    ok = O.label_windows(d, 10, wall=tot + tot // 25)          # 4 % residual: under 5 %
+    assert ok.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_DIRECT_EXPOSURE
+    bad = O.label_windows(d, 10, wall=tot + tot // 10)         # 10 % residual
+    assert bad.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_TELEMETRY_LIMITED
+    ovl = O.label_windows(d, 10, wall=tot - tot // 50)         # 2 % overlap > 1 %
+    assert ovl.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_TELEMETRY_LIMITED
+    # a recorded residual stage (stage 2 as "other") carrying 100/420 of the time
+    oth = O.label_windows(d, 10, other_stage=2)
+    assert oth.labels[0] & O.L_TELEMETRY_LIMITED
+
+
+def test_label_role_aware_needed():
+    L = O.label_windows(_intermittent_data_stall(), 10, role=np.array([0, 0, 1, 1]))
+    assert L.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_ROLE_AWARE_NEEDED
+    same = O.label_windows(_intermittent_data_stall(), 10, role=np.array([3, 3, 3, 3]))
+    assert same.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_DIRECT_EXPOSURE
+
+
+def test_label_two_stage_tie():
+    """R=2, S=2, W=10, base 10 ms; even steps r0 data +30, odd steps r0 bwd
+    +30: a alternates (40,10)/(10,40), X=(250,250), D=500 -> C_A={0,1};
+    every step is confident with alternating leaders (9 switches of 10);
+    medians of r0 are 10 so Y=(150,150), G=0.3 each (a gain tie)."""
+    d = np.full((10, 2, 2), 10 * U, np.int64)
+    d[0::2, 0, 0] += 30 * U
+    d[1::2, 0, 1] += 30 * U
+    L = O.label_windows(d, 10)
+    assert (L.X[0] == [250 * U, 250 * U]).all() and (L.Y[0] == [150 * U, 150 * U]).all()
+    assert L.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_CO_CRITICAL
+    assert L.amb_mask[0] == 0b11 and L.n_confident[0] == 10 and L.n_switch[0] == 9
+
+
+def test_label_leader_switch_only():
+    """Even steps r0 data +50, odd steps r0 bwd +30 (base 10, R=2, W=10):
+    a = (60,10) / (10,40); X=(350,250), D=600: C_A={data} (gap 100 >= 30),
+    A_data=0.583 high; r0 medians: data {60x5,10x5}->10, bwd {40x5,10x5}->10,
+    so Y=(250,150), G_data=0.417 (direct evidence), C_G={data} (gap 100).
+    All 10 steps are confident and alternate -> high switch -> co_critical,
+    and direct_exposure is downgraded."""
+    d = np.full((10, 2, 2), 10 * U, np.int64)
+    d[0::2, 0, 0] += 50 * U
+    d[1::2, 0, 1] += 30 * U
+    L = O.label_windows(d, 10)
+    assert (L.X[0] == [350 * U, 250 * U]).all() and L.D[0] == 600 * U
+    assert (L.Y[0] == [250 * U, 150 * U]).all()
+    assert L.n_switch[0] == 9
+    assert L.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_CO_CRITICAL
+    assert L.amb_mask[0] == 0b01
+
+
+def test_label_raw_only_zero_window():
+    L = O.label_windows(np.zeros((5, 3, 4), np.int64), 5)
+    assert L.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_TELEMETRY_LIMITED | O.L_RAW_ONLY
+    assert L.route_mask[0] == 0 and L.amb_mask[0] == 0 and (L.share == 0).all()
+
+
+def test_label_partial_last_window():
+    d = np.concatenate([_intermittent_data_stall(), np.full((3, 4, 3), 10 * U, np.int64)])
+    L = O.label_windows(d, 10)
+    assert L.labels.shape == (2,)
+    # last window: 3 identical steps, three-way share tie, no confident leader
+    assert L.labels[1] == O.L_FRONTIER_ACCOUNTING | O.L_CO_CRITICAL
+    assert L.amb_mask[1] == 0b111 and L.n_confident[1] == 0
