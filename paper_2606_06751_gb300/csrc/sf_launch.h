@@ -1,0 +1,63 @@
+// sf_launch.h - host-side interface between the C ABI layer (sf_api.cu) and
+// the kernel translation units.  Internal to libstagefrontier.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "stagefrontier.h"
+
+namespace sf {
+
+// Everything a streaming pass over d needs; unused outputs are null.
+struct StreamJob {
+  const int64_t* d = nullptr;
+  int64_t T = 0, R = 0, S = 0;
+  // sf_frontier outputs
+  int64_t* a = nullptr;
+  int32_t* lead = nullptr;
+  int64_t* mk = nullptr;
+  // sf_window_aggregate outputs (and the evidence pass's X / D)
+  int64_t* X = nullptr;
+  int64_t* D = nullptr;
+  int64_t* E = nullptr;
+  int32_t* C = nullptr;
+  uint8_t* step_lead = nullptr;
+  int64_t t0 = 0, W = 1;
+  // evidence pass (sf_direct_gain)
+  bool gain = false;
+  const int64_t* m = nullptr;
+  const int64_t* wall = nullptr;
+  int32_t other_stage = -1;
+  int64_t eta_num = 0, eta_den = 1;
+  int64_t* Y = nullptr;
+  uint64_t* quality = nullptr;
+  uint32_t* status = nullptr;
+};
+
+int sm_count();                     // SMs of the current device (cached)
+void count_launch(uint64_t n = 1);  // bump the library's launch counter
+
+cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t stream);
+cudaError_t launch_stream_pass(const StreamJob& job, cudaStream_t stream);
+cudaError_t launch_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W,
+                                 int64_t* m, cudaStream_t stream);
+cudaError_t launch_topk(const int64_t* X, const int64_t* E, int64_t nW, int64_t S, int64_t R,
+                        int32_t k, int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair,
+                        int64_t* top_pair_value, cudaStream_t stream);
+
+struct GateJob {
+  int64_t T, R, S, W, nW;
+  const int64_t *X, *Y, *D;
+  const uint8_t* step_lead;
+  const uint64_t* quality;
+  const int32_t* role;
+  const int32_t* missing;
+  sf_label_config cfg;
+  uint32_t *labels, *route_mask, *amb_mask;
+  double *share, *gain;
+  int32_t *n_confident, *n_switch;
+};
+cudaError_t launch_gates(const GateJob& job, cudaStream_t stream);
+
+}  // namespace sf

@@ -1,0 +1,408 @@
+// sf_select.cu - the per-window kernels of libstagefrontier:
+//   * window_median: lower median of every (window, rank, stage) column
+//     (the per-rank window baseline of Sec. 4, Eq. 3);
+//   * topk: top-k stages by X and (stage, rank) pairs by lead-rank credit E;
+//   * gates: App. C label gates, routing and ambiguity sets, fp64 shares/gains;
+//   * zero: clears accumulators the library owns the semantics of.
+#include <algorithm>
+
+#include "sf_device.cuh"
+#include "sf_launch.h"
+
+namespace sf {
+
+namespace {
+
+__device__ __forceinline__ int64_t imin64(int64_t a, int64_t b) { return a < b ? a : b; }
+
+__global__ void zero_kernel(uint32_t* __restrict__ p, size_t words) {
+  for (size_t i = blockIdx.x * size_t(blockDim.x) + threadIdx.x; i < words;
+       i += size_t(gridDim.x) * blockDim.x)
+    p[i] = 0u;
+}
+
+// ---------------------------------------------------------------------------
+// Lower median, one warp per column.  A CTA of 8 warps owns (window w, eight
+// consecutive flat columns c = r*S + s).  The window's rows of those columns
+// are read coalesced and transposed through shared memory so each warp holds
+// its column in registers (NPL values per lane).  Selection is a bitwise
+// search on the offset from the column minimum: the k-th smallest value
+// (k = floor((n-1)/2)) is the largest v with #{x < v} <= k, found one bit at
+// a time from the top bit of (max - min), each bit costing one warp-wide
+// count.  Values are compared as signed int64 (mapped to an order-preserving
+// unsigned key), so the result is exact for any input.
+constexpr int kMedCols = 8;
+constexpr int kMedThreads = kMedCols * 32;
+
+template <int NPL>
+__global__ void __launch_bounds__(kMedThreads)
+    median_kernel(const int64_t* __restrict__ d, int64_t T, int64_t RS, int64_t W, int64_t ngroups,
+                  int64_t* __restrict__ m) {
+  constexpr int LD = 32 * NPL + 1;
+  extern __shared__ int64_t colbuf[];  // [kMedCols][LD]
+  const int64_t w = blockIdx.x / ngroups;
+  const int64_t c0 = (blockIdx.x % ngroups) * kMedCols;
+  const int ncols = static_cast<int>(imin64(kMedCols, RS - c0));
+  const int64_t tb = w * W;
+  const int n = static_cast<int>(imin64(W, T - tb));
+  const int64_t* base = d + tb * RS + c0;
+  for (int idx = threadIdx.x; idx < n * kMedCols; idx += kMedThreads) {
+    const int row = idx / kMedCols, c = idx % kMedCols;
+    colbuf[c * LD + row] = c < ncols ? __ldg(base + int64_t(row) * RS + c) : 0;
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (warp >= ncols) return;
+  constexpr uint64_t kSign = 1ull << 63;
+  uint64_t u[NPL];
+  uint64_t lo = ~0ull, hi = 0;
+#pragma unroll
+  for (int i = 0; i < NPL; ++i) {
+    const int row = lane + 32 * i;
+    if (row < n) {
+      u[i] = static_cast<uint64_t>(colbuf[warp * LD + row]) ^ kSign;
+      lo = u[i] < lo ? u[i] : lo;
+      hi = u[i] > hi ? u[i] : hi;
+    } else {
+      u[i] = ~0ull;  // padding sorts after every real value
+    }
+  }
+  lo = warp_min_u64(lo);
+  hi = warp_max_u64(hi);
+  const uint32_t k = static_cast<uint32_t>((n - 1) / 2);
+  const uint64_t range = hi - lo;
+  const int nbits = range ? 64 - __clzll(static_cast<long long>(range)) : 0;
+  uint64_t ans = 0;
+  if (nbits <= 32) {
+    uint32_t x[NPL];
+#pragma unroll
+    for (int i = 0; i < NPL; ++i) {
+      const uint64_t off = u[i] - lo;
+      x[i] = off > 0xffffffffull ? 0xffffffffu : static_cast<uint32_t>(off);
+    }
+    uint32_t a32 = 0;
+    for (int bit = nbits - 1; bit >= 0; --bit) {
+      const uint32_t cand = a32 | (1u << bit);
+      uint32_t cnt = 0;
+#pragma unroll
+      for (int i = 0; i < NPL; ++i) cnt += x[i] < cand ? 1u : 0u;
+      cnt = __reduce_add_sync(kFull, cnt);
+      if (cnt <= k) a32 = cand;
+    }
+    ans = a32;
+  } else {
+    for (int bit = nbits - 1; bit >= 0; --bit) {
+      const uint64_t cand = ans | (1ull << bit);
+      uint32_t cnt = 0;
+#pragma unroll
+      for (int i = 0; i < NPL; ++i) cnt += (u[i] - lo) < cand ? 1u : 0u;
+      cnt = __reduce_add_sync(kFull, cnt);
+      if (cnt <= k) ans = cand;
+    }
+  }
+  if (lane == 0) m[w * RS + c0 + warp] = static_cast<int64_t>((lo + ans) ^ kSign);
+}
+
+// Windows longer than 1024 steps: the same search, re-reading the column
+// from global memory (L2) on every bit.
+__global__ void __launch_bounds__(kMedThreads)
+    median_global_kernel(const int64_t* __restrict__ d, int64_t T, int64_t RS, int64_t W,
+                         int64_t ngroups, int64_t* __restrict__ m) {
+  const int64_t w = blockIdx.x / ngroups;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t c = (blockIdx.x % ngroups) * kMedCols + warp;
+  if (c >= RS) return;
+  const int64_t tb = w * W;
+  const int64_t n = imin64(W, T - tb);
+  const int64_t* col = d + tb * RS + c;
+  constexpr uint64_t kSign = 1ull << 63;
+  uint64_t lo = ~0ull, hi = 0;
+  for (int64_t t = lane; t < n; t += 32) {
+    const uint64_t u = static_cast<uint64_t>(__ldg(col + t * RS)) ^ kSign;
+    lo = u < lo ? u : lo;
+    hi = u > hi ? u : hi;
+  }
+  lo = warp_min_u64(lo);
+  hi = warp_max_u64(hi);
+  const uint64_t k = static_cast<uint64_t>((n - 1) / 2);
+  const uint64_t range = hi - lo;
+  const int nbits = range ? 64 - __clzll(static_cast<long long>(range)) : 0;
+  uint64_t ans = 0;
+  for (int bit = nbits - 1; bit >= 0; --bit) {
+    const uint64_t cand = ans | (1ull << bit);
+    uint32_t cnt = 0;
+    for (int64_t t = lane; t < n; t += 32)
+      cnt += ((static_cast<uint64_t>(__ldg(col + t * RS)) ^ kSign) - lo) < cand ? 1u : 0u;
+    cnt = __reduce_add_sync(kFull, cnt);
+    if (cnt <= k) ans = cand;
+  }
+  if (lane == 0) m[w * RS + c] = static_cast<int64_t>((lo + ans) ^ kSign);
+}
+
+// ---------------------------------------------------------------------------
+// Top-k.  One CTA per window.  Order: value descending, then index ascending
+// (index = stage for X, s*R + r for E); value 0 is not a suspect.
+constexpr int kTopThreads = 256;
+
+struct VI {
+  int64_t v;
+  int64_t i;
+};
+
+__device__ __forceinline__ bool before(const VI& a, const VI& b) {  // a ranks ahead of b
+  return a.v > b.v || (a.v == b.v && a.i < b.i);
+}
+
+__device__ VI block_best(VI x, VI* sm) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    VI y{__shfl_xor_sync(kFull, x.v, o), __shfl_xor_sync(kFull, x.i, o)};
+    if (before(y, x)) x = y;
+  }
+  if (lane == 0) sm[warp] = x;
+  __syncthreads();
+  VI r = sm[0];
+  for (int i = 1; i < kTopThreads / 32; ++i)
+    if (before(sm[i], r)) r = sm[i];
+  __syncthreads();
+  return r;
+}
+
+__global__ void __launch_bounds__(kTopThreads)
+    topk_kernel(const int64_t* __restrict__ X, const int64_t* __restrict__ E, int64_t S, int64_t R,
+                int k, int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair,
+                int64_t* top_pair_value) {
+  __shared__ VI sm[kTopThreads / 32];
+  const int64_t w = blockIdx.x;
+  if (threadIdx.x < 32 && (top_stage || top_stage_value)) {
+    const int lane = threadIdx.x;
+    const int64_t v = lane < S ? X[w * S + lane] : 0;
+    bool taken = false;
+    for (int i = 0; i < k; ++i) {
+      const uint64_t cand = (!taken && lane < S && v > 0) ? static_cast<uint64_t>(v) : 0ull;
+      const uint64_t mx = warp_max_u64(cand);
+      int who = -1;
+      if (mx != 0) who = __ffs(__ballot_sync(kFull, cand == mx)) - 1;  // lowest stage among equals
+      if (lane == who) taken = true;
+      if (lane == 0) {
+        if (top_stage) top_stage[w * k + i] = who;
+        if (top_stage_value) top_stage_value[w * k + i] = who >= 0 ? static_cast<int64_t>(mx) : 0;
+      }
+    }
+  }
+  if (E == nullptr || (top_pair == nullptr && top_pair_value == nullptr)) return;
+  const int64_t n = S * R;
+  const int64_t* Ew = E + w * n;
+  VI prev{INT64_MAX, -1};
+  for (int i = 0; i < k; ++i) {
+    VI best{0, INT64_MAX};
+    for (int64_t j = threadIdx.x; j < n; j += kTopThreads) {
+      const VI c{Ew[j], j};
+      if (c.v <= 0 || !before(prev, c)) continue;  // only entries ranked after the last pick
+      if (before(c, best)) best = c;
+    }
+    best = block_best(best, sm);
+    if (threadIdx.x == 0) {
+      const bool ok = best.v > 0;
+      if (top_pair) {
+        top_pair[(w * k + i) * 2 + 0] = ok ? static_cast<int32_t>(best.i / R) : -1;
+        top_pair[(w * k + i) * 2 + 1] = ok ? static_cast<int32_t>(best.i % R) : -1;
+      }
+      if (top_pair_value) top_pair_value[w * k + i] = ok ? best.v : 0;
+    }
+    if (best.v <= 0) {
+      for (int ii = i + 1 + threadIdx.x; ii < k; ii += kTopThreads) {
+        if (top_pair) top_pair[(w * k + ii) * 2 + 0] = top_pair[(w * k + ii) * 2 + 1] = -1;
+        if (top_pair_value) top_pair_value[w * k + ii] = 0;
+      }
+      break;
+    }
+    prev = best;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Gates (App. C).  One CTA per window: the CTA scans rank roles and splits the
+// window's step leaders into 256 segments for the switch count; thread 0 then
+// evaluates the gates with exact integer comparisons a*den <op> num*b.
+constexpr int kGateThreads = 256;
+
+__device__ __forceinline__ bool r_gt(__int128 lhs, sf_ratio r, __int128 rhs) {
+  return lhs * r.den > static_cast<__int128>(r.num) * rhs;
+}
+__device__ __forceinline__ bool r_lt(__int128 lhs, sf_ratio r, __int128 rhs) {
+  return lhs * r.den < static_cast<__int128>(r.num) * rhs;
+}
+__device__ __forceinline__ bool r_ge(__int128 lhs, sf_ratio r, __int128 rhs) {
+  return lhs * r.den >= static_cast<__int128>(r.num) * rhs;
+}
+
+__global__ void __launch_bounds__(kGateThreads) gates_kernel(const GateJob g) {
+  __shared__ int seg_e[kGateThreads], seg_sw[kGateThreads], seg_first[kGateThreads],
+      seg_last[kGateThreads];
+  const int64_t w = blockIdx.x;
+  const int64_t S = g.S;
+  const int64_t tb = w * g.W, te = min(tb + g.W, g.T), n = te - tb;
+  int mixed = 0;
+  if (g.role) {
+    const int32_t r0 = g.role[0];
+    for (int64_t r = 1 + threadIdx.x; r < g.R; r += kGateThreads) mixed |= g.role[r] != r0;
+  }
+  mixed = __syncthreads_or(mixed);
+  {
+    const int j = threadIdx.x;
+    const int64_t sb = tb + n * j / kGateThreads, se = tb + n * (j + 1) / kGateThreads;
+    int e = 0, sw = 0, first = -1, last = -1;
+    for (int64_t t = sb; t < se; ++t) {
+      const uint8_t sl = g.step_lead[t];
+      if (sl & SF_STEP_CONFIDENT) {
+        const int ld = sl & 31;
+        if (last >= 0 && ld != last) ++sw;
+        if (first < 0) first = ld;
+        last = ld;
+        ++e;
+      }
+    }
+    seg_e[j] = e;
+    seg_sw[j] = sw;
+    seg_first[j] = first;
+    seg_last[j] = last;
+  }
+  __syncthreads();
+  if (threadIdx.x != 0) return;
+
+  int64_t e = 0, sw = 0;
+  int last = -1;
+  for (int j = 0; j < kGateThreads; ++j) {
+    if (seg_e[j] == 0) continue;
+    e += seg_e[j];
+    sw += seg_sw[j] + ((last >= 0 && seg_first[j] != last) ? 1 : 0);
+    last = seg_last[j];
+  }
+  const sf_label_config& c = g.cfg;
+  const bool high_switch = e >= 2 && r_ge(e, c.gamma_elig, n) && r_gt(sw, c.gamma_switch, e - 1);
+
+  const int64_t* Xw = g.X + w * S;
+  const int64_t* Yw = g.Y + w * S;
+  const int64_t Dw = g.D[w];
+  bool tel = g.missing != nullptr && g.missing[w] > c.max_missing_ranks;
+  if (g.quality) {
+    const uint64_t* q = g.quality + w * 6;
+    const unsigned __int128 res = (static_cast<unsigned __int128>(q[1]) << 64) | q[0];
+    const unsigned __int128 ovl = (static_cast<unsigned __int128>(q[3]) << 64) | q[2];
+    const unsigned __int128 ws = (static_cast<unsigned __int128>(q[5]) << 64) | q[4];
+    if (res * static_cast<uint64_t>(c.closure_max.den) > ws * static_cast<uint64_t>(c.closure_max.num)) tel = true;
+    if (ovl * static_cast<uint64_t>(c.overlap_max.den) > ws * static_cast<uint64_t>(c.overlap_max.num)) tel = true;
+  }
+  const bool raw = Dw < c.denom_floor_ns || Dw == 0;
+  if (raw) tel = true;
+  uint32_t lab = SF_LABEL_FRONTIER_ACCOUNTING, route = 0, amb = 0;
+  if (tel) lab |= SF_LABEL_TELEMETRY_LIMITED;
+  if (mixed) lab |= SF_LABEL_ROLE_AWARE_NEEDED;
+  if (raw) {
+    lab |= SF_LABEL_RAW_ONLY;
+  } else {
+    int s1 = 0, g1 = 0;
+    for (int s = 1; s < S; ++s) {
+      if (Xw[s] > Xw[s1]) s1 = s;
+      if (Yw[s] > Yw[g1]) g1 = s;
+    }
+    int nA = 0, nG = 0;
+    for (int s = 0; s < S; ++s) {
+      if (r_lt(Xw[s1] - Xw[s], c.eta_A, Dw)) {
+        amb |= 1u << s;
+        ++nA;
+      }
+      if (r_lt(Yw[g1] - Yw[s], c.eta_G, Dw)) {
+        amb |= 1u << s;
+        ++nG;
+      }
+    }
+    __int128 cum = 0;
+    for (int i = 0; i < S; ++i) {  // leading-share prefix reaching tau_C
+      int pick = -1;
+      for (int s = 0; s < S; ++s)
+        if (!((route >> s) & 1u) && (pick < 0 || Xw[s] > Xw[pick])) pick = s;
+      route |= 1u << pick;
+      cum += Xw[pick];
+      if (r_ge(cum, c.tau_C, Dw)) break;
+    }
+    const bool hiA = r_gt(Xw[s1], c.gamma_A, Dw);
+    const bool loG = r_lt(Yw[s1], c.gamma_G, Dw);
+    const bool W1 = (c.model_fit_mask >> s1) & 1u;
+    const bool gain_tie = nG >= 2 && r_ge(Yw[g1], c.gamma_G, Dw);
+    if (hiA && loG) lab |= W1 ? SF_LABEL_SYNC_WAIT_DEPENDENT : SF_LABEL_CO_CRITICAL;
+    if (hiA && !loG) lab |= SF_LABEL_DIRECT_EXPOSURE;
+    if (nA >= 2 || gain_tie || high_switch) {
+      lab |= SF_LABEL_CO_CRITICAL;
+      lab &= ~(SF_LABEL_DIRECT_EXPOSURE | SF_LABEL_SYNC_WAIT_DEPENDENT);
+    }
+    if (tel || mixed) lab &= ~(SF_LABEL_DIRECT_EXPOSURE | SF_LABEL_SYNC_WAIT_DEPENDENT);
+  }
+  g.labels[w] = lab;
+  g.route_mask[w] = route;
+  g.amb_mask[w] = amb;
+  for (int s = 0; s < S; ++s) {
+    if (g.share) g.share[w * S + s] = raw ? 0.0 : static_cast<double>(Xw[s]) / static_cast<double>(Dw);
+    if (g.gain) g.gain[w * S + s] = raw ? 0.0 : static_cast<double>(Yw[s]) / static_cast<double>(Dw);
+  }
+  if (g.n_confident) g.n_confident[w] = static_cast<int32_t>(e);
+  if (g.n_switch) g.n_switch[w] = static_cast<int32_t>(sw);
+}
+
+template <int NPL>
+cudaError_t launch_median_npl(const int64_t* d, int64_t T, int64_t RS, int64_t W, int64_t nW,
+                              int64_t ngroups, int64_t* m, cudaStream_t stream) {
+  const size_t smem = size_t(kMedCols) * (32 * NPL + 1) * sizeof(int64_t);
+  cudaError_t e = cudaFuncSetAttribute(median_kernel<NPL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  median_kernel<NPL><<<static_cast<unsigned>(nW * ngroups), kMedThreads, smem, stream>>>(d, T, RS, W, ngroups, m);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t stream) {
+  if (bytes == 0) return cudaSuccess;
+  const size_t words = bytes / 4;
+  const int grid = static_cast<int>(std::min<size_t>((words + 255) / 256, size_t(sm_count()) * 8));
+  count_launch();
+  zero_kernel<<<grid, 256, 0, stream>>>(static_cast<uint32_t*>(p), words);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W,
+                                 int64_t* m, cudaStream_t stream) {
+  const int64_t RS = R * S;
+  const int64_t nW = (T + W - 1) / W;
+  const int64_t ngroups = (RS + kMedCols - 1) / kMedCols;
+  const int64_t n = std::min(W, T);
+  count_launch();
+  if (n <= 32) return launch_median_npl<1>(d, T, RS, W, nW, ngroups, m, stream);
+  if (n <= 64) return launch_median_npl<2>(d, T, RS, W, nW, ngroups, m, stream);
+  if (n <= 128) return launch_median_npl<4>(d, T, RS, W, nW, ngroups, m, stream);
+  if (n <= 256) return launch_median_npl<8>(d, T, RS, W, nW, ngroups, m, stream);
+  if (n <= 512) return launch_median_npl<16>(d, T, RS, W, nW, ngroups, m, stream);
+  if (n <= 1024) return launch_median_npl<32>(d, T, RS, W, nW, ngroups, m, stream);
+  median_global_kernel<<<static_cast<unsigned>(nW * ngroups), kMedThreads, 0, stream>>>(d, T, RS, W, ngroups, m);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_topk(const int64_t* X, const int64_t* E, int64_t nW, int64_t S, int64_t R, int32_t k,
+                        int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair,
+                        int64_t* top_pair_value, cudaStream_t stream) {
+  count_launch();
+  topk_kernel<<<static_cast<unsigned>(nW), kTopThreads, 0, stream>>>(X, E, S, R, k, top_stage, top_stage_value,
+                                                                     top_pair, top_pair_value);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gates(const GateJob& job, cudaStream_t stream) {
+  count_launch();
+  gates_kernel<<<static_cast<unsigned>(job.nW), kGateThreads, 0, stream>>>(job);
+  return cudaGetLastError();
+}
+
+}  // namespace sf

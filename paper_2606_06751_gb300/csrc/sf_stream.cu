@@ -1,0 +1,754 @@
+// sf_stream.cu - the streaming passes over the telemetry tensor d[T][R][S]:
+//
+//   * frontier pass (Sec. 3 Eq. 1-2): rank-local prefixes in registers, the
+//     max-prefix frontier with its lowest attaining rank per boundary, the
+//     increments a[t,s], and the fused window aggregation (X, D, E, C, leading
+//     stage);
+//   * evidence pass (Sec. 4 Eq. 3): the same frontier plus, for every stage s,
+//     the makespan after replacing s by the clipped per-rank window median,
+//     per-step leader confidence and the telemetry-quality sums (App. A).
+//
+// Fast path (S even, S <= 16, R*S a multiple of 16): a persistent grid, one
+// CTA per SM, each CTA owning a contiguous range of steps.  One producer
+// thread streams 128-byte rows of d into a ring of shared-memory tiles with 2-D
+// bulk tensor copies (TMA) completing on mbarriers; eight consumer warps read
+// whole rank rows out of the tiles (128B-swizzled when S/2 is a power of two,
+// which makes the strided 16-byte row reads bank-conflict free), keep the
+// prefix and per-boundary maxima in registers, and reduce across ranks with
+// warp redux plus one shared-memory exchange.  Small steps (<= 16 KB) are
+// handled one step per warp with several steps per tile; large steps one step
+// per CTA spread over several tiles.
+//
+// Generic path (any other S <= 32 or R): one CTA per step range with plain
+// global loads.  Both paths share the per-step epilogues.
+#include <algorithm>
+#include <numeric>
+
+#include "sf_device.cuh"
+#include "sf_launch.h"
+
+namespace sf {
+
+namespace {
+
+constexpr int kConsumerWarps = 8;
+constexpr int kConsumerThreads = kConsumerWarps * 32;
+constexpr int kBlockThreads = kConsumerThreads + 32;  // + one producer warp
+constexpr int kRowBytes = 128;                        // TMA row: 16 int64
+constexpr int kMaxBoxRows = 256;
+constexpr int kTileBytes = kMaxBoxRows * kRowBytes;   // 32 KB per ring stage
+constexpr int kStages = 6;
+constexpr int kRedSlots = 2 * kConsumerWarps * 32;    // double-buffered per-warp partials
+constexpr size_t kSmemBytes = 1024 /*alignment slack*/ + size_t(kStages) * kTileBytes +
+                              2 * kStages * sizeof(uint64_t) + 16 + kRedSlots * sizeof(uint64_t);
+
+struct Params {
+  int64_t T, R, S;
+  int64_t step_rows;  // 128-byte rows per step
+  int regime;         // 0: several steps per tile, 1: tiles per step
+  int box_rows, K, tiles_per_step;
+  int64_t* a;
+  int32_t* lead;
+  int64_t* mk;
+  int64_t* X;
+  int64_t* D;
+  int64_t* E;
+  int32_t* C;
+  uint8_t* step_lead;
+  int64_t t0, W, w_first;
+  const int64_t* m;
+  const int64_t* wall;
+  int other_stage;
+  int64_t eta_num, eta_den;
+  int64_t* Y;
+  uint64_t* quality;
+  uint32_t* status;
+};
+
+__device__ __forceinline__ uint32_t hi32(int64_t v) {
+  return static_cast<uint32_t>(static_cast<uint64_t>(v) >> 32);
+}
+
+// --------------------------------------------------------------------------
+// Window accumulators held by the warp that finalizes steps: lane s keeps the
+// stage-s numerators, every lane the denominator.
+struct WinAcc {
+  int64_t cur = -1;
+  int64_t x = 0, y = 0, dsum = 0;
+};
+
+__device__ __forceinline__ void flush_window(const Params& p, int S, WinAcc& acc, int lane) {
+  if (acc.cur >= 0) {
+    if (lane < S) {
+      if (acc.x) atomicAdd(reinterpret_cast<unsigned long long*>(&p.X[acc.cur * S + lane]),
+                           static_cast<unsigned long long>(acc.x));
+      if (p.Y && acc.y)
+        atomicAdd(reinterpret_cast<unsigned long long*>(&p.Y[acc.cur * S + lane]),
+                  static_cast<unsigned long long>(acc.y));
+    }
+    if (lane == 0 && acc.dsum)
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.D[acc.cur]),
+                static_cast<unsigned long long>(acc.dsum));
+  }
+  acc.x = acc.y = acc.dsum = 0;
+}
+
+// Frontier epilogue for step t.  Lane s < S holds the packed key
+// (F[t,s] << 16) | (65535 - lead[t,s]); the whole warp participates.
+__device__ __forceinline__ void finalize_frontier(const Params& p, int S, int64_t t, uint64_t key,
+                                                  int lane, WinAcc& acc) {
+  const bool valid = lane < S;
+  const int64_t F = valid ? static_cast<int64_t>(key >> 16) : 0;
+  const int32_t ld = valid ? 65535 - static_cast<int32_t>(key & 0xffffu) : 0;
+  int64_t Fprev = __shfl_up_sync(kFull, F, 1);
+  if (lane == 0) Fprev = 0;  // F[t,-1] = 0
+  const int64_t a = valid ? F - Fprev : 0;
+  const int64_t mk = __shfl_sync(kFull, F, S - 1);
+  if (valid) {
+    if (p.a) p.a[t * S + lane] = a;
+    if (p.lead) p.lead[t * S + lane] = ld;
+  }
+  if (lane == 0 && p.mk) p.mk[t] = mk;
+  if (p.X) {
+    const int64_t w = (p.t0 + t) / p.W - p.w_first;
+    if (w != acc.cur) {
+      flush_window(p, S, acc, lane);
+      acc.cur = w;
+    }
+    acc.x += a;
+    acc.dsum += mk;
+    if (valid && ld >= 0 && ld < p.R) {  // always true for valid input; guards flagged input
+      const int64_t idx = (w * S + lane) * p.R + ld;
+      if (p.E && a != 0)
+        atomicAdd(reinterpret_cast<unsigned long long*>(&p.E[idx]), static_cast<unsigned long long>(a));
+      if (p.C) atomicAdd(&p.C[idx], 1);
+    }
+    if (p.step_lead) {
+      const uint64_t k2 = valid ? ((static_cast<uint64_t>(a) << 5) | static_cast<uint64_t>(31 - lane)) : 0;
+      const uint64_t km = warp_max_u64(k2);
+      if (lane == 0) p.step_lead[t] = static_cast<uint8_t>(31 - static_cast<int>(km & 31u));
+    }
+  }
+}
+
+// Evidence epilogue for step t.  Lane s < S holds F[t,s] and
+// Fr[t,s] = max_r (P[t,r,S-1] - max(0, d[t,r,s] - m[w,r,s])).
+__device__ __forceinline__ void finalize_gain(const Params& p, int S, int64_t t, int64_t F,
+                                              int64_t Fr, int lane, WinAcc& acc) {
+  const bool valid = lane < S;
+  int64_t Fprev = __shfl_up_sync(kFull, F, 1);
+  if (lane == 0) Fprev = 0;
+  const int64_t a = valid ? F - Fprev : 0;
+  const int64_t FS = __shfl_sync(kFull, F, S - 1);
+  const int64_t y = valid ? FS - Fr : 0;
+  // leading stage (largest increment, lowest stage) and the runner-up increment
+  const uint64_t k2 = valid ? ((static_cast<uint64_t>(a) << 5) | static_cast<uint64_t>(31 - lane)) : 0;
+  const uint64_t km = warp_max_u64(k2);
+  const int best = 31 - static_cast<int>(km & 31u);
+  const int64_t amax = static_cast<int64_t>(km >> 5);
+  const int64_t second = static_cast<int64_t>(warp_max_u64(valid && lane != best ? static_cast<uint64_t>(a) : 0));
+  const bool conf = FS > 0 && static_cast<__int128>(amax - second) * p.eta_den >=
+                                  static_cast<__int128>(p.eta_num) * FS;
+  if (lane == 0) p.step_lead[t] = static_cast<uint8_t>(best | (conf ? SF_STEP_CONFIDENT : 0u));
+  const int64_t w = t / p.W;
+  if (w != acc.cur) {
+    flush_window(p, S, acc, lane);
+    acc.cur = w;
+  }
+  acc.x += a;
+  acc.y += y;
+  acc.dsum += FS;
+}
+
+// Telemetry-quality sums of one thread (App. A closure / overlap), flushed per window.
+struct QualAcc {
+  int64_t cur = -1;
+  unsigned __int128 res = 0, ovl = 0, wsum = 0;
+};
+
+__device__ __forceinline__ unsigned __int128 warp_sum_u128(unsigned __int128 v) {
+  uint64_t lo = static_cast<uint64_t>(v), hi = static_cast<uint64_t>(v >> 64);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const uint64_t olo = __shfl_xor_sync(kFull, lo, o);
+    const uint64_t ohi = __shfl_xor_sync(kFull, hi, o);
+    const uint64_t nlo = lo + olo;
+    hi = hi + ohi + (nlo < lo ? 1u : 0u);
+    lo = nlo;
+  }
+  return (static_cast<unsigned __int128>(hi) << 64) | lo;
+}
+
+// Warp-uniform: every lane calls with the same window index w.
+__device__ __forceinline__ void qual_window(const Params& p, QualAcc& q, int64_t w, int lane) {
+  if (w == q.cur) return;
+  if (q.cur >= 0) {
+    const unsigned __int128 r = warp_sum_u128(q.res), o = warp_sum_u128(q.ovl), s = warp_sum_u128(q.wsum);
+    if (lane == 0) {
+      uint64_t* dst = p.quality + q.cur * 6;
+      if (r) atomic_add_u128(dst + 0, r);
+      if (o) atomic_add_u128(dst + 2, o);
+      if (s) atomic_add_u128(dst + 4, s);
+    }
+  }
+  q.res = q.ovl = q.wsum = 0;
+  q.cur = w;
+}
+
+__device__ __forceinline__ void qual_row(const Params& p, QualAcc& q, int64_t t, int64_t r,
+                                         int64_t total, int64_t other, uint32_t& dor) {
+  if (p.wall) {
+    const int64_t wv = p.wall[t * p.R + r];
+    dor |= hi32(wv);
+    const int64_t e = wv - (total - other);  // e = w - sum_{s != other} d
+    if (e > 0) q.res += static_cast<uint64_t>(e);
+    else q.ovl += static_cast<uint64_t>(-e);
+    q.wsum += static_cast<uint64_t>(wv);
+  } else {
+    q.res += static_cast<uint64_t>(other);
+    q.wsum += static_cast<uint64_t>(total);
+  }
+}
+
+// --------------------------------------------------------------------------
+// Per-thread running maxima over the rank rows a thread visits (in increasing
+// rank order, so a strict '>' keeps the lowest rank on ties).
+template <int S>
+struct FrontierRows {
+  int64_t bp[S];
+  int32_t br[S];
+  __device__ __forceinline__ void init() {
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      bp[s] = -1;
+      br[s] = 0;
+    }
+  }
+  __device__ __forceinline__ void row(const int64_t (&v)[S], int32_t r, uint32_t& dor, uint32_t& tor) {
+    int64_t P = 0;
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      dor |= hi32(v[s]);
+      P += v[s];  // P[t,r,s]
+      if (P > bp[s]) {
+        bp[s] = P;
+        br[s] = r;
+      }
+    }
+    tor |= hi32(P);
+  }
+  __device__ __forceinline__ uint64_t key(int s) const {
+    return bp[s] < 0 ? 0ull
+                     : (static_cast<uint64_t>(bp[s]) << 16) | static_cast<uint64_t>(65535 - br[s]);
+  }
+};
+
+template <int S>
+struct GainRows {
+  int64_t bf[S];  // max_r P[t,r,s]
+  int64_t bg[S];  // max_r (P[t,r,S-1] - max(0, d[t,r,s] - m[w,r,s]))
+  __device__ __forceinline__ void init() {
+#pragma unroll
+    for (int s = 0; s < S; ++s) bf[s] = bg[s] = 0;
+  }
+  __device__ __forceinline__ int64_t row(const int64_t (&v)[S], const int64_t (&mr)[S], uint32_t& dor,
+                                         uint32_t& tor) {
+    int64_t P = 0;
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      dor |= hi32(v[s]);
+      P += v[s];
+      bf[s] = P > bf[s] ? P : bf[s];
+    }
+    tor |= hi32(P);
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      int64_t cut = v[s] - mr[s];
+      cut = cut > 0 ? cut : 0;
+      const int64_t alt = P - cut;
+      bg[s] = alt > bg[s] ? alt : bg[s];
+    }
+    return P;
+  }
+};
+
+template <int S>
+__device__ __forceinline__ int64_t pick(const int64_t (&v)[S], int idx) {
+  int64_t o = 0;
+#pragma unroll
+  for (int s = 0; s < S; ++s) o = (s == idx) ? v[s] : o;
+  return o;
+}
+
+// Read rank row q (S int64) of a tile; the 16-byte chunk c of the tile lives
+// at physical chunk c ^ ((c >> 3) & 7) when the tile was written with the
+// 128-byte swizzle.
+template <int S, bool kSwz>
+__device__ __forceinline__ void load_row(const unsigned char* tile, int q, int64_t (&v)[S]) {
+  constexpr int M = S / 2;
+  const int c0 = q * M;
+#pragma unroll
+  for (int j = 0; j < M; ++j) {
+    const int c = c0 + j;
+    const int pc = kSwz ? (c ^ ((c >> 3) & 7)) : c;
+    const longlong2 x = *reinterpret_cast<const longlong2*>(tile + pc * 16);
+    v[2 * j] = x.x;
+    v[2 * j + 1] = x.y;
+  }
+}
+
+template <int S>
+__device__ __forceinline__ void load_global_row(const int64_t* src, int64_t (&v)[S]) {
+#pragma unroll
+  for (int j = 0; j < S / 2; ++j) {
+    const longlong2 x = __ldg(reinterpret_cast<const longlong2*>(src) + j);
+    v[2 * j] = x.x;
+    v[2 * j + 1] = x.y;
+  }
+}
+
+// Offset the dynamic shared-memory base to the next 1024-byte boundary (the
+// 128-byte swizzle pattern repeats every 1024 bytes); pointer arithmetic keeps
+// the shared address space visible to the compiler.
+__device__ __forceinline__ unsigned char* align_1024(unsigned char* p) {
+  return p + ((1024u - (smem_u32(p) & 1023u)) & 1023u);
+}
+
+// Wait (bounded, ignoring abort) for copies still in flight before the CTA exits.
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return;
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity))
+    if (global_timer_ns() - t0 > kWaitLimitNs) return;
+}
+
+__device__ void produce(const CUtensorMap* map, const Params& p, int64_t t_begin, int64_t t_end,
+                        unsigned char* ring, uint64_t* full, uint64_t* empty, volatile int* abort) {
+  prefetch_tensormap(map);
+  const uint32_t bytes = static_cast<uint32_t>(p.box_rows) * kRowBytes;
+  uint32_t j = 0;
+  bool ok = true;
+  auto issue = [&](int64_t row) {
+    const uint32_t st = j % kStages, ph = (j / kStages) & 1u;
+    if (!mbar_wait_bounded(&empty[st], ph ^ 1u, abort)) {
+      ok = false;
+      return;
+    }
+    mbar_arrive_expect_tx(&full[st], bytes);
+    tma_load_2d(ring + size_t(st) * kTileBytes, map, 0, static_cast<int32_t>(row), &full[st]);
+    ++j;
+  };
+  if (p.regime == 0) {
+    for (int64_t t = t_begin; t < t_end && ok; t += p.K) issue(t * p.step_rows);
+  } else {
+    for (int64_t t = t_begin; t < t_end && ok; ++t)
+      for (int k = 0; k < p.tiles_per_step && ok; ++k) {
+        const int64_t r0 = min(int64_t(k) * p.box_rows, p.step_rows - p.box_rows);
+        issue(t * p.step_rows + r0);
+      }
+  }
+  for (uint32_t i = j > uint32_t(kStages) ? j - kStages : 0; i < j; ++i)
+    drain_wait(&full[i % kStages], (i / kStages) & 1u);
+}
+
+// --------------------------------------------------------------------------
+template <int S, bool GAIN>
+__global__ void __launch_bounds__(kBlockThreads, 1)
+    stream_kernel(const __grid_constant__ CUtensorMap map, const Params p) {
+  constexpr bool kSwz = (S == 4 || S == 8 || S == 16);
+  constexpr int U = S <= 8 ? 4 : 2;  // rank rows in flight per thread
+  constexpr int NV = GAIN ? 2 * S : S;
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* ring = align_1024(smem_raw);
+  uint64_t* full = reinterpret_cast<uint64_t*>(ring + size_t(kStages) * kTileBytes);
+  uint64_t* empty = full + kStages;
+  volatile int* abort = reinterpret_cast<volatile int*>(empty + kStages);
+  uint64_t* red = reinterpret_cast<uint64_t*>(empty + kStages) + 2;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t G = gridDim.x, b = blockIdx.x;
+  const int64_t t_begin = p.T * b / G, t_end = p.T * (b + 1) / G;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], p.regime == 0 ? static_cast<uint32_t>(p.K) : uint32_t(kConsumerWarps));
+    }
+    *abort = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+
+  if (warp == kConsumerWarps) {
+    if (lane == 0) produce(&map, p, t_begin, t_end, ring, full, empty, abort);
+    return;
+  }
+
+  uint32_t dor = 0, tor = 0;  // OR of duration / rank-total high words
+  WinAcc acc;
+  QualAcc qa;
+  const int R = static_cast<int>(p.R);
+
+  if (p.regime == 0) {
+    // ---- one step per warp, K steps per tile
+    const int64_t n_local = t_end - t_begin;
+    for (int64_t i = warp; i < n_local; i += kConsumerWarps) {
+      const uint32_t j = static_cast<uint32_t>(i / p.K);
+      const uint32_t st = j % kStages, ph = (j / kStages) & 1u;
+      const bool have = mbar_wait_bounded(&full[st], ph, abort);
+      const int kk = static_cast<int>(i - int64_t(j) * p.K);
+      const unsigned char* tile = ring + size_t(st) * kTileBytes;
+      const int64_t t = t_begin + i;
+      const int64_t w = GAIN ? t / p.W : 0;
+      if (GAIN && p.quality) qual_window(p, qa, w, lane);
+      const int q0 = kk * R;
+      if constexpr (!GAIN) {
+        FrontierRows<S> rs;
+        rs.init();
+        if (have) {
+          for (int r0 = lane; r0 < R; r0 += 32 * U) {
+            int64_t v[U][S];
+#pragma unroll
+            for (int u = 0; u < U; ++u)
+              if (r0 + 32 * u < R) load_row<S, kSwz>(tile, q0 + r0 + 32 * u, v[u]);
+#pragma unroll
+            for (int u = 0; u < U; ++u)
+              if (r0 + 32 * u < R) rs.row(v[u], r0 + 32 * u, dor, tor);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[st]);
+        uint64_t mykey = 0;
+#pragma unroll
+        for (int s = 0; s < S; ++s) {
+          const uint64_t km = warp_max_u64(rs.key(s));
+          if (lane == s) mykey = km;
+        }
+        finalize_frontier(p, S, t, mykey, lane, acc);
+      } else {
+        GainRows<S> rs;
+        rs.init();
+        if (have) {
+          for (int r = lane; r < R; r += 32) {
+            int64_t v[S], mr[S];
+            load_row<S, kSwz>(tile, q0 + r, v);
+            load_global_row<S>(p.m + (w * p.R + r) * S, mr);
+            const int64_t total = rs.row(v, mr, dor, tor);
+            if (p.quality)
+              qual_row(p, qa, t, r, total, p.other_stage >= 0 ? pick<S>(v, p.other_stage) : 0, dor);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[st]);
+        int64_t myF = 0, myR = 0;
+#pragma unroll
+        for (int s = 0; s < S; ++s) {
+          const uint64_t f = warp_max_u64(static_cast<uint64_t>(rs.bf[s]));
+          const uint64_t g = warp_max_u64(static_cast<uint64_t>(rs.bg[s]));
+          if (lane == s) {
+            myF = static_cast<int64_t>(f);
+            myR = static_cast<int64_t>(g);
+          }
+        }
+        finalize_gain(p, S, t, myF, myR, lane, acc);
+      }
+    }
+  } else {
+    // ---- one step per CTA, tiles_per_step tiles per step
+    const int ctid = threadIdx.x;
+    uint32_t j = 0;
+    int buf = 0;
+    for (int64_t t = t_begin; t < t_end; ++t) {
+      const int64_t w = GAIN ? t / p.W : 0;
+      if (GAIN && p.quality) qual_window(p, qa, w, lane);
+      FrontierRows<S> fr;
+      GainRows<S> gr;
+      if constexpr (GAIN) gr.init(); else fr.init();
+      for (int k = 0; k < p.tiles_per_step; ++k, ++j) {
+        const uint32_t st = j % kStages, ph = (j / kStages) & 1u;
+        const bool have = mbar_wait_bounded(&full[st], ph, abort);
+        const unsigned char* tile = ring + size_t(st) * kTileBytes;
+        const int64_t row0 = min(int64_t(k) * p.box_rows, p.step_rows - p.box_rows);
+        const int rank_tile0 = static_cast<int>(row0 * 16 / S);
+        const int rank_fresh = static_cast<int>(int64_t(k) * p.box_rows * 16 / S);
+        const int rank_end = static_cast<int>((row0 + p.box_rows) * 16 / S);
+        if (have) {
+          if constexpr (!GAIN) {
+            for (int r0 = rank_fresh + ctid; r0 < rank_end; r0 += kConsumerThreads * U) {
+              int64_t v[U][S];
+#pragma unroll
+              for (int u = 0; u < U; ++u)
+                if (r0 + kConsumerThreads * u < rank_end)
+                  load_row<S, kSwz>(tile, r0 + kConsumerThreads * u - rank_tile0, v[u]);
+#pragma unroll
+              for (int u = 0; u < U; ++u)
+                if (r0 + kConsumerThreads * u < rank_end) fr.row(v[u], r0 + kConsumerThreads * u, dor, tor);
+            }
+          } else {
+            for (int r = rank_fresh + ctid; r < rank_end; r += kConsumerThreads) {
+              int64_t v[S], mr[S];
+              load_row<S, kSwz>(tile, r - rank_tile0, v);
+              load_global_row<S>(p.m + (w * p.R + r) * S, mr);
+              const int64_t total = gr.row(v, mr, dor, tor);
+              if (p.quality)
+                qual_row(p, qa, t, r, total, p.other_stage >= 0 ? pick<S>(v, p.other_stage) : 0, dor);
+            }
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[st]);
+      }
+      // cross-rank reduction: warp redux, then one exchange through shared memory
+      uint64_t* slot = red + (buf * kConsumerWarps + warp) * 32;
+#pragma unroll
+      for (int s = 0; s < S; ++s) {
+        if constexpr (!GAIN) {
+          const uint64_t km = warp_max_u64(fr.key(s));
+          if (lane == s) slot[s] = km;
+        } else {
+          const uint64_t f = warp_max_u64(static_cast<uint64_t>(gr.bf[s]));
+          const uint64_t g = warp_max_u64(static_cast<uint64_t>(gr.bg[s]));
+          if (lane == s) {
+            slot[s] = f;
+            slot[S + s] = g;
+          }
+        }
+      }
+      named_barrier(1, kConsumerThreads);
+      if (warp == 0) {
+        uint64_t v0 = 0, v1 = 0;
+        if (lane < S) {
+#pragma unroll
+          for (int ww = 0; ww < kConsumerWarps; ++ww) {
+            const uint64_t* sl = red + (buf * kConsumerWarps + ww) * 32;
+            v0 = sl[lane] > v0 ? sl[lane] : v0;
+            if (GAIN) v1 = sl[S + lane] > v1 ? sl[S + lane] : v1;
+          }
+        }
+        if constexpr (!GAIN) finalize_frontier(p, S, t, v0, lane, acc);
+        else finalize_gain(p, S, t, static_cast<int64_t>(v0), static_cast<int64_t>(v1), lane, acc);
+      }
+      buf ^= 1;
+    }
+    (void)NV;
+  }
+
+  if (p.X && (p.regime == 0 || warp == 0)) flush_window(p, S, acc, lane);
+  if (GAIN && p.quality) qual_window(p, qa, -2, lane);
+  const uint32_t bits = range_bits(__reduce_or_sync(kFull, dor), __reduce_or_sync(kFull, tor)) |
+                        (*abort ? SF_ST_TIMEOUT : 0u);
+  if (lane == 0) report(p.status, bits);
+}
+
+// --------------------------------------------------------------------------
+// Generic path: any S <= 32, any R; one CTA of 256 threads per step range.
+constexpr int kGenThreads = 256;
+
+template <bool GAIN>
+__global__ void __launch_bounds__(kGenThreads)
+    stream_generic_kernel(const int64_t* __restrict__ d, const Params p) {
+  __shared__ uint64_t red[kGenThreads / 32][64];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int S = static_cast<int>(p.S);
+  const int64_t R = p.R;
+  const int64_t G = gridDim.x, b = blockIdx.x;
+  const int64_t t_begin = p.T * b / G, t_end = p.T * (b + 1) / G;
+  uint32_t dor = 0, tor = 0;
+  WinAcc acc;
+  QualAcc qa;
+  for (int64_t t = t_begin; t < t_end; ++t) {
+    const int64_t w = GAIN ? t / p.W : 0;
+    if (GAIN && p.quality) qual_window(p, qa, w, lane);
+    int64_t b0[32], b1[32];
+    int32_t br[32];
+    for (int s = 0; s < S; ++s) {
+      b0[s] = GAIN ? 0 : -1;
+      b1[s] = 0;
+      br[s] = 0;
+    }
+    for (int64_t r = threadIdx.x; r < R; r += kGenThreads) {
+      const int64_t* row = d + (t * R + r) * S;
+      int64_t P = 0, other = 0;
+      for (int s = 0; s < S; ++s) {
+        const int64_t v = row[s];
+        dor |= hi32(v);
+        P += v;
+        if (s == p.other_stage) other = v;
+        if (P > b0[s]) {
+          b0[s] = P;
+          br[s] = static_cast<int32_t>(r);
+        }
+      }
+      tor |= hi32(P);
+      if (GAIN) {
+        const int64_t* mr = p.m + (w * R + r) * S;
+        for (int s = 0; s < S; ++s) {
+          int64_t cut = row[s] - mr[s];
+          cut = cut > 0 ? cut : 0;
+          b1[s] = (P - cut) > b1[s] ? (P - cut) : b1[s];
+        }
+        if (p.quality) qual_row(p, qa, t, r, P, other, dor);
+      }
+    }
+    for (int s = 0; s < S; ++s) {
+      uint64_t k0;
+      if (GAIN) k0 = static_cast<uint64_t>(b0[s]);
+      else k0 = b0[s] < 0 ? 0ull : (static_cast<uint64_t>(b0[s]) << 16) | static_cast<uint64_t>(65535 - br[s]);
+      const uint64_t m0 = warp_max_u64(k0);
+      const uint64_t m1 = GAIN ? warp_max_u64(static_cast<uint64_t>(b1[s])) : 0;
+      if (lane == 0) {
+        red[warp][s] = m0;
+        red[warp][32 + s] = m1;
+      }
+    }
+    __syncthreads();
+    if (warp == 0) {
+      uint64_t v0 = 0, v1 = 0;
+      if (lane < S)
+        for (int ww = 0; ww < kGenThreads / 32; ++ww) {
+          v0 = red[ww][lane] > v0 ? red[ww][lane] : v0;
+          v1 = red[ww][32 + lane] > v1 ? red[ww][32 + lane] : v1;
+        }
+      if (GAIN) finalize_gain(p, S, t, static_cast<int64_t>(v0), static_cast<int64_t>(v1), lane, acc);
+      else finalize_frontier(p, S, t, v0, lane, acc);
+    }
+    __syncthreads();
+  }
+  if (p.X && warp == 0) flush_window(p, S, acc, lane);
+  if (GAIN && p.quality) qual_window(p, qa, -2, lane);
+  const uint32_t bits = range_bits(__reduce_or_sync(kFull, dor), __reduce_or_sync(kFull, tor));
+  if (lane == 0) report(p.status, bits);
+}
+
+// --------------------------------------------------------------------------
+// Host side
+using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                              const cuuint64_t*, const cuuint32_t*, const cuuint32_t*,
+                              CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                              CUtensorMapFloatOOBfill);
+
+EncodeFn encode_fn() {
+  static EncodeFn fn = [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      f = nullptr;
+    return reinterpret_cast<EncodeFn>(f);
+  }();
+  return fn;
+}
+
+template <int S, bool GAIN>
+cudaError_t prepare_fast() {
+  return cudaFuncSetAttribute(stream_kernel<S, GAIN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(kSmemBytes));
+}
+
+template <bool GAIN>
+cudaError_t dispatch_fast(int S, const CUtensorMap& map, const Params& p, int grid, cudaStream_t stream) {
+#define SF_CASE(SV)                                                                          \
+  case SV: {                                                                                 \
+    cudaError_t e = prepare_fast<SV, GAIN>();                                     \
+    if (e != cudaSuccess) return e;                                                          \
+    stream_kernel<SV, GAIN><<<grid, kBlockThreads, kSmemBytes, stream>>>(map, p);            \
+    return cudaGetLastError();                                                               \
+  }
+  switch (S) {
+    SF_CASE(2)
+    SF_CASE(4)
+    SF_CASE(6)
+    SF_CASE(8)
+    SF_CASE(10)
+    SF_CASE(12)
+    SF_CASE(14)
+    SF_CASE(16)
+    default:
+      return cudaErrorInvalidValue;
+  }
+#undef SF_CASE
+}
+
+}  // namespace
+
+cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
+  Params p{};
+  p.T = j.T;
+  p.R = j.R;
+  p.S = j.S;
+  p.a = j.a;
+  p.lead = j.lead;
+  p.mk = j.mk;
+  p.X = j.X;
+  p.D = j.D;
+  p.E = j.E;
+  p.C = j.C;
+  p.step_lead = j.step_lead;
+  p.t0 = j.t0;
+  p.W = j.W;
+  p.w_first = j.t0 / j.W;
+  p.m = j.m;
+  p.wall = j.wall;
+  p.other_stage = j.other_stage;
+  p.eta_num = j.eta_num;
+  p.eta_den = j.eta_den;
+  p.Y = j.Y;
+  p.quality = j.quality;
+  p.status = j.status;
+
+  const int64_t RS = j.R * j.S;
+  const int64_t step_rows = RS / 16;
+  const int64_t rows_total = j.T * step_rows;
+  const bool fast = (j.S % 2 == 0) && j.S <= 16 && (RS % 16 == 0) &&
+                    rows_total <= int64_t(0x7fffffff) && encode_fn() != nullptr &&
+                    (reinterpret_cast<uintptr_t>(j.d) % 16 == 0) &&
+                    (!j.gain || reinterpret_cast<uintptr_t>(j.m) % 16 == 0);
+  const int sms = sm_count();
+  if (fast) {
+    p.step_rows = step_rows;
+    if (step_rows <= kMaxBoxRows / 2) {
+      p.regime = 0;
+      p.K = static_cast<int>(kMaxBoxRows / step_rows);
+      p.box_rows = static_cast<int>(p.K * step_rows);
+      p.tiles_per_step = 0;
+    } else {
+      p.regime = 1;
+      // rows per rank-aligned block: a tile must hold whole rank rows
+      const int64_t elems = 16 * j.S / std::gcd<int64_t>(16, j.S);  // lcm(16, S)
+      const int64_t q = elems / 16;
+      int64_t n = (step_rows + kMaxBoxRows - 1) / kMaxBoxRows, br = 0;
+      for (;; ++n) {
+        br = (step_rows + n - 1) / n;
+        br = (br + q - 1) / q * q;
+        if (br <= kMaxBoxRows) break;
+      }
+      p.box_rows = static_cast<int>(br);
+      p.tiles_per_step = static_cast<int>((step_rows + br - 1) / br);
+      p.K = 0;
+    }
+    CUtensorMap map;
+    const cuuint64_t gdim[2] = {16, static_cast<cuuint64_t>(rows_total)};
+    const cuuint64_t gstride[1] = {kRowBytes};
+    const cuuint32_t box[2] = {16, static_cast<cuuint32_t>(p.box_rows)};
+    const cuuint32_t estride[2] = {1, 1};
+    const bool swz = (j.S == 4 || j.S == 8 || j.S == 16);
+    CUresult cr = encode_fn()(&map, CU_TENSOR_MAP_DATA_TYPE_INT64, 2, const_cast<int64_t*>(j.d), gdim,
+                              gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                              swz ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    const int64_t units = p.regime == 0 ? (j.T + p.K - 1) / p.K : j.T;
+    const int grid = static_cast<int>(std::min<int64_t>(sms, units));
+    count_launch();
+    return j.gain ? dispatch_fast<true>(static_cast<int>(j.S), map, p, grid, stream)
+                  : dispatch_fast<false>(static_cast<int>(j.S), map, p, grid, stream);
+  }
+  const int grid = static_cast<int>(std::min<int64_t>(int64_t(sms) * 4, j.T));
+  count_launch();
+  if (j.gain) stream_generic_kernel<true><<<grid, kGenThreads, 0, stream>>>(j.d, p);
+  else stream_generic_kernel<false><<<grid, kGenThreads, 0, stream>>>(j.d, p);
+  return cudaGetLastError();
+}
+
+}  // namespace sf

@@ -1,0 +1,248 @@
+"""GPU parity: every output of the CUDA path against the CPU oracle, element
+by element, on seeded inputs that span several tiles, ragged tails, both
+streaming regimes and the generic path.  Integer outputs must be bit-exact;
+fp64 shares/gains within 1e-12 relative (they are one IEEE division of the
+same integers, so equality is expected)."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as O
+from synth import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+RTOL = 1e-12
+
+
+@pytest.fixture(scope="module")
+def sf():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_06751_gb300 import build as B
+    B.build()
+    from paper_2606_06751_gb300 import stagefrontier
+    return stagefrontier
+
+
+def dev(x):
+    return torch.from_numpy(np.ascontiguousarray(x)).cuda()
+
+
+def host(t):
+    return t.cpu().numpy()
+
+
+def make(T, R, S, seed, kind):
+    rng = np.random.default_rng(seed)
+    if kind == "ties":      # tiny value range: ties at almost every boundary
+        return rng.integers(0, 6, size=(T, R, S), dtype=np.int64)
+    if kind == "zeros":     # many zero durations and equal prefixes
+        d = rng.integers(0, 1000, size=(T, R, S), dtype=np.int64)
+        d[rng.random((T, R, S)) < 0.6] = 0
+        return d
+    # lognormal around ms medians with one sync stage (realistic skew)
+    med = rng.uniform(1e6, 5e7, size=S)
+    x = np.rint(med * np.exp(0.1 * rng.standard_normal((T, R, S)))).astype(np.int64)
+    return x
+
+
+# (T, R, S): generic path; fast path one-step-per-warp (<= 16 KB steps);
+# fast path one-step-per-CTA with overlapped last tile.
+SHAPES = [
+    (37, 3, 5), (20, 1, 1), (11, 7, 32), (9, 65, 3), (6, 5, 18),          # generic
+    (1000, 8, 6), (301, 128, 8), (123, 64, 4), (77, 64, 16), (50, 2, 8),   # one step per warp
+    (301, 16, 2), (97, 40, 10), (45, 24, 14), (33, 120, 12),
+    (13, 1024, 10), (7, 8192, 8), (5, 4096, 16), (3, 32768, 4),            # one step per CTA
+    (9, 520, 12), (6, 1000, 14), (4, 512, 8), (3, 65536, 2),
+]
+
+
+@pytest.mark.parametrize("T,R,S", SHAPES)
+@pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal"])
+def test_frontier_parity(sf, T, R, S, kind):
+    d_np = make(T, R, S, T * 131 + R * 7 + S, kind)
+    o = O.frontier(d_np)
+    st = sf.new_status("cuda")
+    f = sf.sf_frontier(dev(d_np), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert np.array_equal(host(f.a), o.a)
+    assert np.array_equal(host(f.lead), o.lead)
+    assert np.array_equal(host(f.makespan), o.makespan)
+
+
+@pytest.mark.parametrize("T,R,S", SHAPES[:4] + SHAPES[5:9] + SHAPES[14:18])
+@pytest.mark.parametrize("t0,W", [(0, 7), (13, 10), (0, 1000)])
+def test_window_aggregate_parity(sf, T, R, S, t0, W):
+    d_np = make(T, R, S, T + R + S + t0, "ties" if R < 100 else "lognormal")
+    o = O.windows(d_np, W, t0)
+    st = sf.new_status("cuda")
+    g = sf.sf_window_aggregate(dev(d_np), W, t0=t0, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    for name in ("X", "D", "E", "C", "step_lead"):
+        assert np.array_equal(host(getattr(g, name)), getattr(o, name)), name
+
+
+def test_window_aggregate_chunked_accumulate(sf):
+    T, R, S, W, chunk = 90, 64, 8, 25, 35
+    d_np = make(T, R, S, 5, "lognormal")
+    o = O.windows(d_np, W, 0)
+    d = dev(d_np)
+    nW = sf.num_windows(0, T, W)
+    X = torch.zeros((nW, S), dtype=torch.int64, device="cuda")
+    D = torch.zeros(nW, dtype=torch.int64, device="cuda")
+    E = torch.zeros((nW, S, R), dtype=torch.int64, device="cuda")
+    C = torch.zeros((nW, S, R), dtype=torch.int32, device="cuda")
+    for t0 in range(0, T, chunk):
+        w0 = t0 // W
+        n = min(chunk, T - t0)
+        sf.sf_window_aggregate(d[t0:t0 + n], W, t0=t0, X=X[w0:], D=D[w0:], E=E[w0:], C=C[w0:],
+                               want=(), accumulate=True)
+    assert np.array_equal(host(X), o.X) and np.array_equal(host(D), o.D)
+    assert np.array_equal(host(E), o.E) and np.array_equal(host(C), o.C)
+
+
+@pytest.mark.parametrize("nW,S,R,k", [(3, 5, 7, 6), (4, 8, 128, 2), (2, 10, 1024, 5), (1, 32, 3, 32),
+                                      (5, 1, 1, 3)])
+def test_topk_parity(sf, nW, S, R, k):
+    rng = np.random.default_rng(nW * S * R)
+    X = rng.integers(0, 4, size=(nW, S)).astype(np.int64)
+    E = rng.integers(0, 4, size=(nW, S, R)).astype(np.int64)
+    o = O.topk(X, E, k)
+    t = sf.sf_topk_suspects(dev(X), dev(E), k)
+    assert np.array_equal(host(t.stage), o.stage) and np.array_equal(host(t.stage_value), o.stage_value)
+    assert np.array_equal(host(t.pair), o.pair) and np.array_equal(host(t.pair_value), o.pair_value)
+
+
+@pytest.mark.parametrize("T,R,S,W", [(100, 8, 6, 100), (250, 4, 3, 32), (130, 5, 4, 64), (300, 2, 8, 128),
+                                     (700, 3, 2, 256), (1100, 2, 4, 512), (2100, 1, 4, 1000),
+                                     (2200, 2, 2, 1024), (2500, 1, 3, 1100), (45, 1024, 10, 20)])
+@pytest.mark.parametrize("kind", ["ties", "lognormal", "wide"])
+def test_median_parity(sf, T, R, S, W, kind):
+    if kind == "wide":  # signed values spanning more than 2^32: the 64-bit search path
+        rng = np.random.default_rng(T + W)
+        d_np = rng.integers(-(1 << 40), 1 << 40, size=(T, R, S), dtype=np.int64)
+    else:
+        d_np = make(T, R, S, T + W, kind)
+    o = O.window_median(d_np, W)
+    m = sf.sf_window_median(dev(d_np), W)
+    assert np.array_equal(host(m), o)
+
+
+@pytest.mark.parametrize("T,R,S,W", [(120, 8, 6, 50), (64, 128, 8, 30), (40, 1024, 10, 16),
+                                     (33, 3, 5, 10), (20, 8192, 8, 8), (30, 64, 16, 30)])
+def test_direct_gain_parity(sf, T, R, S, W):
+    d_np = make(T, R, S, R + S, "lognormal")
+    m_np = O.window_median(d_np, W)
+    Y = O.direct_gain(d_np, W, m_np)
+    ow = O.windows(d_np, W)
+    ev = sf.sf_direct_gain(dev(d_np), W, dev(m_np))
+    assert np.array_equal(host(ev.Y), Y)
+    assert np.array_equal(host(ev.D), [ow.D[w] for w in range(len(ow.D))])
+    assert np.array_equal(host(ev.X), ow.X)
+    assert np.array_equal(host(ev.step_lead) & 31, ow.step_lead)
+
+
+def compare_labels(sf, d_np, W, role=None, missing=None, wall=None, other_stage=-1, cfg=None):
+    o = O.label_windows(d_np, W, role=role, missing=missing, wall=wall, other_stage=other_stage, cfg=cfg)
+    args = {}
+    for name, v in (("role", role), ("missing", missing), ("wall", wall)):
+        if v is not None:
+            args[name] = dev(v)
+    cfg_sf = None
+    if cfg is not None:
+        cfg_sf = sf.default_config()
+        cfg_sf.model_fit_mask = cfg.model_fit_mask
+    st = sf.new_status("cuda")
+    lab = sf.sf_label_windows(dev(d_np), W, other_stage=other_stage, cfg=cfg_sf, status=st, **args)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert np.array_equal(host(lab.labels).astype(np.uint32), o.labels)
+    assert np.array_equal(host(lab.route_mask).astype(np.uint32), o.route_mask)
+    assert np.array_equal(host(lab.amb_mask).astype(np.uint32), o.amb_mask)
+    assert np.array_equal(host(lab.X), o.X) and np.array_equal(host(lab.Y), o.Y)
+    assert np.array_equal(host(lab.D), o.D)
+    np.testing.assert_allclose(host(lab.share), o.share, rtol=RTOL, atol=0)
+    np.testing.assert_allclose(host(lab.gain), o.gain, rtol=RTOL, atol=0)
+    # the gates entry point also reports the leader-switch evidence
+    ev = sf.sf_direct_gain(dev(d_np), W, sf.sf_window_median(dev(d_np), W))
+    g = sf.sf_label_gates(d_np.shape[0], d_np.shape[1], d_np.shape[2], W, ev)
+    assert np.array_equal(host(g.n_confident), o.n_confident)
+    assert np.array_equal(host(g.n_switch), o.n_switch)
+    return o
+
+
+U = 1_000_000
+
+
+def test_label_fixtures(sf):
+    base = np.full((10, 4, 3), 10 * U, np.int64)
+    base[0:4, 0, 0] += 30 * U                                     # intermittent data stall
+    o = compare_labels(sf, base, 10)
+    assert o.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_DIRECT_EXPOSURE
+    compare_labels(sf, base, 10, missing=np.array([1], np.int32))
+    compare_labels(sf, base, 10, role=np.array([0, 0, 1, 1], np.int32))
+    tot = base.sum(axis=2)
+    compare_labels(sf, base, 10, wall=tot + tot // 10)
+    compare_labels(sf, base, 10, wall=tot - tot // 50)
+    compare_labels(sf, base, 10, other_stage=2)
+    sharp = np.repeat(np.array([[[10, 0], [0, 10]]], np.int64) * 10**9, 20, axis=0)
+    o = compare_labels(sf, sharp, 20)
+    assert o.labels[0] == O.L_FRONTIER_ACCOUNTING | O.L_CO_CRITICAL and o.amb_mask[0] == 3
+    cfg = O.default_config()
+    cfg.model_fit_mask = 1
+    compare_labels(sf, sharp, 20, cfg=cfg)
+    tie = np.full((10, 2, 2), 10 * U, np.int64)
+    tie[0::2, 0, 0] += 30 * U
+    tie[1::2, 0, 1] += 30 * U
+    compare_labels(sf, tie, 10)
+    compare_labels(sf, np.zeros((5, 3, 4), np.int64), 5)
+    compare_labels(sf, np.concatenate([base, np.full((3, 4, 3), 10 * U, np.int64)]), 10)
+
+
+@pytest.mark.parametrize("name,steps", [("tiny", None), ("ddp128", 3000), ("fsdp1024", 1000),
+                                        ("accum8192", 60)])
+def test_labels_on_workloads(sf, name, steps):
+    w = wl.by_name(name, steps=steps)
+    d_np = w.generate()
+    W = min(w.W, max(1, steps // 3)) if steps else w.W
+    rng = np.random.default_rng(1)
+    missing = (rng.random((d_np.shape[0] + W - 1) // W) < 0.3).astype(np.int32)
+    compare_labels(sf, d_np, W)
+    compare_labels(sf, d_np, W, missing=missing, wall=w.wall(d_np), other_stage=w.S - 1)
+
+
+def test_device_status_bits(sf):
+    d_np = np.ones((16, 64, 8), np.int64)
+    d_np[3, 5, 2] = -4
+    st = sf.new_status("cuda")
+    sf.sf_frontier(dev(d_np), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & sf.SF_ST_NEGATIVE
+    d_np[3, 5, 2] = 1 << 47
+    st.zero_()
+    sf.sf_window_aggregate(dev(d_np), 4, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & sf.SF_ST_RANGE
+    d_np[3, 5, 2] = 1 << 46
+    d_np[3, 5, 3] = 1 << 46                          # rank total reaches 2^47
+    st.zero_()
+    sf.sf_frontier(dev(d_np), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == sf.SF_ST_RANGE
+    d_np = np.ones((16, 3, 5), np.int64)             # generic path
+    d_np[0, 0, 0] = -1
+    st.zero_()
+    sf.sf_frontier(dev(d_np), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & sf.SF_ST_NEGATIVE
+
+
+def test_deterministic_repeat(sf):
+    d = dev(make(200, 256, 8, 3, "ties"))
+    a = sf.sf_window_aggregate(d, 50)
+    b = sf.sf_window_aggregate(d, 50)
+    for name in ("X", "D", "E", "C", "step_lead"):
+        assert torch.equal(getattr(a, name), getattr(b, name))
