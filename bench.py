@@ -1,0 +1,433 @@
+"""Benchmark of the frontier-accounting hot path on GB300.
+
+One step = one pass of the whole path over one batch of synthetic telemetry:
+window aggregation fused into the frontier pass (Sec. 3 Eq. 1-2), top-k
+suspects, and the labeler (per-rank window medians, the clipped-gain evidence
+pass of Sec. 4 Eq. 3, App. C gates).  The default workload is the largest
+frontier-accounting configuration: 8192 ranks x 8 stages x 20000 steps of
+int64 ns (10.49 GB), 1000-step windows, top-5, labels.
+
+Prints ONE JSON line (rank 0).  `value` is rank.step.stage records per
+second with the input resident in HBM (CUDA events on the launching stream,
+max over ranks); `e2e` is the same metric through the library's public API
+with the input in pinned host memory and its host->device copy (plus the
+device->host read of the results) inside the timed region.  `roofline` is
+the dominant kernel's algorithmic HBM bytes over its event-timed duration
+against the measured copy bandwidth.  `cpu_baseline` times the CPU oracle on
+a bounded sample of the same workload.
+
+Multi-GPU (torchrun): one independent replica per GPU (the path has no
+exchange step), weak scaling, barrier + max-over-ranks timing.
+`--impl reference` times the CPU oracle itself as the reference arm.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from synth import workloads as wl  # noqa: E402
+
+METRIC = "rank·step·stage records/sec and achieved HBM GB/s (% of GB300 peak)"
+UNIT = "records/s"
+KERNEL_SOURCES = ("sf_stream.cu", "sf_select.cu", "sf_device.cuh")
+
+
+# --------------------------------------------------------------------------- distributed harness
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def init_dist(backend: str):
+    ws, rank, _ = dist_env()
+    if ws > 1 and not torch.distributed.is_initialized():
+        torch.distributed.init_process_group(backend=backend)
+    return ws, rank
+
+
+def barrier(ws: int):
+    if ws > 1:
+        torch.distributed.barrier()
+
+
+def max_over_ranks(x: float, ws: int, device) -> float:
+    if ws == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def timed_loop(step, K: int, W: int, ws: int, device, use_cuda: bool) -> float:
+    """Run W untimed then K timed steps; returns the max-over-ranks seconds."""
+    for _ in range(W):
+        step()
+    if use_cuda:
+        torch.cuda.synchronize()
+    barrier(ws)
+    if use_cuda:
+        stream = torch.cuda.current_stream()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(K):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        secs = e0.elapsed_time(e1) / 1e3
+    else:
+        t0 = time.perf_counter()
+        for _ in range(K):
+            step()
+        secs = time.perf_counter() - t0
+    barrier(ws)
+    return max_over_ranks(secs, ws, device)
+
+
+# --------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu = gpu_id
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_gpu{os.getpid()}.csv")
+
+    def __enter__(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------- helpers
+
+def smi_gpu_id(local: int) -> str:
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        ids = [v.strip() for v in vis.split(",") if v.strip()]
+        if local < len(ids):
+            return ids[local]
+    return str(local)
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def kernel_source_sha() -> str:
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2606_06751_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch recorded from an ncu capture in profiles/, valid
+    only while the kernel sources are unchanged (matching source sha)."""
+    sha = kernel_source_sha()
+    pdir = os.path.join(ROOT, "profiles")
+    if not os.path.isdir(pdir):
+        return None
+    for fn in sorted(os.listdir(pdir)):
+        if not fn.endswith(".md"):
+            continue
+        txt = open(os.path.join(pdir, fn)).read()
+        for m in re.finditer(r"traffic_per_launch\s+kernel=(\S+)\s+workload=(\S+)\s+bytes=(\d+)\s+"
+                             r"source_sha=(\S+)", txt):
+            if m.group(1) == kernel and m.group(2) == workload and m.group(4) == sha:
+                return int(m.group(3))
+    return None
+
+
+# --------------------------------------------------------------------------- our arm
+
+class Pipeline:
+    """Device buffers and the per-step sequence of library calls."""
+
+    def __init__(self, sf, w: wl.Workload, d: torch.Tensor):
+        self.sf, self.w, self.d = sf, w, d
+        dev = d.device
+        T, R, S, W, k = w.T, w.R, w.S, w.W, w.k
+        self.nW = sf.num_windows(0, T, W)
+        nW = self.nW
+        e = lambda shape, dt: torch.empty(shape, dtype=dt, device=dev)  # noqa: E731
+        self.win = sf.Windows(e((nW, S), torch.int64), e((nW,), torch.int64), e((nW, S, R), torch.int64),
+                              e((nW, S, R), torch.int32), e((T,), torch.uint8))
+        self.top = sf.TopK(e((nW, k), torch.int32), e((nW, k), torch.int64), e((nW, k, 2), torch.int32),
+                           e((nW, k), torch.int64))
+        self.m = e((nW, R, S), torch.int64)
+        self.ev = sf.Evidence(e((nW, S), torch.int64), e((nW, S), torch.int64), e((nW,), torch.int64),
+                              e((T,), torch.uint8), None)
+        self.lab = sf.Labels(e((nW,), torch.int32), e((nW,), torch.int32), e((nW,), torch.int32),
+                             e((nW, S), torch.float64), e((nW, S), torch.float64), e((nW,), torch.int32),
+                             e((nW,), torch.int32))
+        self.status = sf.new_status(dev)
+        self.names = ["window_aggregate", "topk_suspects", "window_median", "direct_gain", "label_gates"]
+        self.events = None
+
+    def step(self, d=None, timing=False):
+        sf, w = self.sf, self.w
+        d = self.d if d is None else d
+        ev = None
+        if timing:
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+            ev[0].record()
+        sf.sf_window_aggregate(d, w.W, X=self.win.X, D=self.win.D, E=self.win.E, C=self.win.C,
+                               step_lead=self.win.step_lead, status=self.status)
+        if timing:
+            ev[1].record()
+        sf.sf_topk_suspects(self.win.X, self.win.E, w.k, out=self.top)
+        if timing:
+            ev[2].record()
+        sf.sf_window_median(d, w.W, m=self.m, status=self.status)
+        if timing:
+            ev[3].record()
+        sf.sf_direct_gain(d, w.W, self.m, out=self.ev, status=self.status)
+        if timing:
+            ev[4].record()
+        sf.sf_label_gates(w.T, w.R, w.S, w.W, self.ev, out=self.lab)
+        if timing:
+            ev[5].record()
+            self.events.append(ev)
+
+    def results(self):
+        return [self.lab.labels, self.lab.route_mask, self.lab.amb_mask, self.lab.share, self.lab.gain,
+                self.top.stage, self.top.pair, self.top.pair_value, self.win.X, self.win.D]
+
+    def algorithmic_bytes(self):
+        w, nW = self.w, self.nW
+        din = w.T * w.R * w.S * 8
+        return {
+            "window_aggregate": din + nW * w.S * (w.R * 12 + 8) + nW * 8 + w.T,
+            "topk_suspects": nW * w.S * (w.R + 1) * 8 + nW * w.k * 24,
+            "window_median": din + nW * w.R * w.S * 8,
+            "direct_gain": din + nW * w.R * w.S * 8 + nW * (2 * w.S + 1) * 8 + w.T,
+            "label_gates": nW * (2 * w.S + 1) * 8 + w.T + nW * (3 * 4 + 2 * w.S * 8),
+        }
+
+
+def run_ours(args):
+    ws, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    init_dist("nccl")
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_06751_gb300 import stagefrontier as sf
+
+    w = wl.by_name(args.workload, seed=args.seed + rank, steps=args.steps_override)
+    host = torch.empty((w.T, w.R, w.S), dtype=torch.int64, pin_memory=True)
+    w.fill(host.numpy().reshape(-1), threads=max(1, (os.cpu_count() or 1) // ws))
+    d = torch.empty_like(host, device=device)
+    d.copy_(host)
+    torch.cuda.synchronize()
+    pipe = Pipeline(sf, w, d)
+    records = w.records
+
+    # device-resident timing, clocks sampled throughout
+    pipe.events = []
+    n0 = sf.launch_count()
+    with ClockSampler(smi_gpu_id(local)) as clk:
+        secs = timed_loop(lambda: pipe.step(timing=True), args.steps, args.warmup, ws, device, True)
+    launches = sf.launch_count() - n0
+    torch.cuda.synchronize()
+    st = int(pipe.status.item())
+    if st != 0:
+        raise RuntimeError(f"device status {st} during the timed region")
+    timed = pipe.events[args.warmup:]
+    per_kernel = {n: [] for n in pipe.names}
+    for ev in timed:
+        for i, n in enumerate(pipe.names):
+            per_kernel[n].append(ev[i].elapsed_time(ev[i + 1]) / 1e3)
+    avg = {n: sum(v) / len(v) for n, v in per_kernel.items()}
+    algo = pipe.algorithmic_bytes()
+    dominant = max(avg, key=avg.get)
+    peak, peak_kind = peaks()
+    achieved = algo[dominant] / avg[dominant] / 1e9
+    value = records * ws * args.steps / secs
+
+    # end to end: pinned host input copied in, results read back, every step
+    outs = pipe.results()
+    host_outs = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
+    d2h = sum(o.numel() * o.element_size() for o in outs)
+
+    def e2e_step():
+        d.copy_(host, non_blocking=True)
+        pipe.step()
+        for h, o in zip(host_outs, outs):
+            h.copy_(o, non_blocking=True)
+
+    e2e_secs = timed_loop(e2e_step, max(3, args.steps // 2), args.warmup, ws, device, True)
+    e2e_value = records * ws * max(3, args.steps // 2) / e2e_secs
+
+    if rank != 0:
+        return None
+    kernels = {n: {"ms": round(avg[n] * 1e3, 4), "gbs": round(algo[n] / avg[n] / 1e9, 1),
+                   "algorithmic_bytes": algo[n]} for n in pipe.names}
+    traffic = profiled_traffic(dominant, w.name)
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+        "config": {"workload": f"{w.name}: {w.R} ranks x {w.S} stages x {w.T} steps int64 ns "
+                               f"({w.nbytes / 1e9:.2f} GB), windows of {w.W}, top-{w.k}, labels",
+                   "R": w.R, "S": w.S, "T": w.T, "W": w.W, "k": w.k, "seed": args.seed,
+                   "l2": f"input {w.nbytes / 1e9:.1f} GB > 129 MB L2 on every pass; no flush",
+                   "parallelism": "replicas" if ws > 1 else "single"},
+        "step_gbs": sum(algo[n] for n in pipe.names) / (secs / args.steps) / 1e9,
+        "roofline": {"kernel": dominant, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+                     "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
+                     "traffic": traffic},
+        "kernels": kernels,
+        "gpu_launches": int(launches * args.steps // (args.steps + args.warmup)),
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": w.nbytes, "d2h_bytes_per_step": d2h},
+        "clocks": clk.summary(),
+    }
+    if ws == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, args.cpu_sample_windows)
+    return line
+
+
+# --------------------------------------------------------------------------- oracle arm
+
+def oracle_step(O, w: wl.Workload, d_np: np.ndarray):
+    """The whole hot path on the CPU oracle, as it stands."""
+    win = O.windows(d_np, w.W)
+    O.topk(win.X, win.E, w.k)
+    O.label_windows(d_np, w.W)
+
+
+def cpu_baseline(w: wl.Workload, n_windows: int):
+    from oracle import oracle as O
+    n = min(w.T, n_windows * w.W)
+    d_np = w.generate(t0=0, nsteps=n)
+    t0 = time.perf_counter()
+    oracle_step(O, w, d_np)
+    secs = time.perf_counter() - t0
+    rec = n * w.R * w.S
+    return {"value": rec / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"first {n} steps ({n // w.W} windows) of {w.name}: {rec} records, "
+                      f"{secs:.1f} s single-threaded C oracle (frontier/windows, top-k, medians, gains, gates)"}
+
+
+def run_reference(args):
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return None
+    from oracle import oracle as O
+    O.build_lib()
+    w = wl.by_name(args.workload, seed=args.seed, steps=args.steps_override)
+    n = min(w.T, args.ref_sample_steps)
+    d_np = w.generate(t0=0, nsteps=n)
+    ww = wl.Workload(**{**w.__dict__, "T": n})
+    for _ in range(args.warmup):
+        oracle_step(O, ww, d_np)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_step(O, ww, d_np)
+    secs = time.perf_counter() - t0
+    rec = n * w.R * w.S
+    value = rec * args.steps / secs
+    sample = (f"each step: first {n} steps of {w.name} ({rec} records; a window shorter than "
+              f"{w.W} steps), single-threaded C oracle")
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+        "data": "synthetic",
+        "config": {"workload": f"{w.name}: {w.R} ranks x {w.S} stages x {w.T} steps int64 ns, "
+                               f"windows of {w.W}, top-{w.k}, labels", "R": w.R, "S": w.S, "T": w.T,
+                   "W": w.W, "k": w.k, "seed": args.seed, "sample_steps": n},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="accum8192")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--steps-override", type=int, default=None, help="shrink T (tests only)")
+    ap.add_argument("--cpu-sample-windows", type=int, default=2)
+    ap.add_argument("--ref-sample-steps", type=int, default=100)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    line = run_reference(args) if args.impl == "reference" else run_ours(args)
+    if line is not None:
+        print(json.dumps(line), flush=True)
+    if torch.distributed.is_initialized():
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

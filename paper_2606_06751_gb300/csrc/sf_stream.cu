@@ -15,9 +15,9 @@
 // whole rank rows out of the tiles (128B-swizzled when S/2 is a power of two,
 // which makes the strided 16-byte row reads bank-conflict free), keep the
 // prefix and per-boundary maxima in registers, and reduce across ranks with
-// warp redux plus one shared-memory exchange.  Small steps (<= 16 KB) are
-// handled one step per warp with several steps per tile; large steps one step
-// per CTA spread over several tiles.
+// warp redux plus one shared-memory exchange.  Small steps (<= 12 KB) are
+// handled by one warp per tile of whole steps, each warp owning two ring
+// stages; large steps one step per CTA spread over several tiles.
 //
 // Generic path (any other S <= 32 or R): one CTA per step range with plain
 // global loads.  Both paths share the per-step epilogues.
@@ -35,12 +35,22 @@ constexpr int kConsumerWarps = 8;
 constexpr int kConsumerThreads = kConsumerWarps * 32;
 constexpr int kBlockThreads = kConsumerThreads + 32;  // + one producer warp
 constexpr int kRowBytes = 128;                        // TMA row: 16 int64
-constexpr int kMaxBoxRows = 256;
-constexpr int kTileBytes = kMaxBoxRows * kRowBytes;   // 32 KB per ring stage
-constexpr int kStages = 6;
+// The 192 KB shared-memory ring is cut two ways.  Small steps (regime 0):
+// 16 stages of 12 KB, two per consumer warp; warp w owns stages 2w and 2w+1
+// and consumes every 8th tile through them in order, so no warp can run a
+// phase ahead of a stage another warp still uses.  Large steps (regime 1):
+// 6 stages of 32 KB that every consumer warp visits in order.
+constexpr int kRingBytes = 192 * 1024;
+constexpr int kR0Stages = 2 * kConsumerWarps;
+constexpr int kR0StageBytes = kRingBytes / kR0Stages;  // 12 KB
+constexpr int kR0MaxRows = kR0StageBytes / kRowBytes;   // 96 rows
+constexpr int kR1Stages = 6;
+constexpr int kR1StageBytes = kRingBytes / kR1Stages;  // 32 KB
+constexpr int kR1MaxRows = kR1StageBytes / kRowBytes;   // 256 rows (the TMA box limit)
+constexpr int kMaxStages = kR0Stages;
 constexpr int kRedSlots = 2 * kConsumerWarps * 32;    // double-buffered per-warp partials
-constexpr size_t kSmemBytes = 1024 /*alignment slack*/ + size_t(kStages) * kTileBytes +
-                              2 * kStages * sizeof(uint64_t) + 16 + kRedSlots * sizeof(uint64_t);
+constexpr size_t kSmemBytes = 1024 /*alignment slack*/ + size_t(kRingBytes) +
+                              2 * kMaxStages * sizeof(uint64_t) + 16 + kRedSlots * sizeof(uint64_t);
 
 struct Params {
   int64_t T, R, S;
@@ -322,20 +332,37 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
     if (global_timer_ns() - t0 > kWaitLimitNs) return;
 }
 
+// Ring stage and phase parity of the j-th tile a CTA streams.
+__device__ __forceinline__ void stage_of(int regime, uint32_t j, uint32_t& st, uint32_t& ph) {
+  if (regime == 0) {  // tile j belongs to warp j % 8, which alternates its two stages
+    const uint32_t i = j / kConsumerWarps;
+    st = 2u * (j % kConsumerWarps) + (i & 1u);
+    ph = (i >> 1) & 1u;
+  } else {
+    st = j % kR1Stages;
+    ph = (j / kR1Stages) & 1u;
+  }
+}
+
+__device__ __forceinline__ size_t stage_bytes(int regime) {
+  return regime == 0 ? size_t(kR0StageBytes) : size_t(kR1StageBytes);
+}
+
 __device__ void produce(const CUtensorMap* map, const Params& p, int64_t t_begin, int64_t t_end,
                         unsigned char* ring, uint64_t* full, uint64_t* empty, volatile int* abort) {
   prefetch_tensormap(map);
   const uint32_t bytes = static_cast<uint32_t>(p.box_rows) * kRowBytes;
-  uint32_t j = 0;
+  uint32_t j = 0;  // tiles issued
   bool ok = true;
   auto issue = [&](int64_t row) {
-    const uint32_t st = j % kStages, ph = (j / kStages) & 1u;
+    uint32_t st, ph;
+    stage_of(p.regime, j, st, ph);
     if (!mbar_wait_bounded(&empty[st], ph ^ 1u, abort)) {
       ok = false;
       return;
     }
     mbar_arrive_expect_tx(&full[st], bytes);
-    tma_load_2d(ring + size_t(st) * kTileBytes, map, 0, static_cast<int32_t>(row), &full[st]);
+    tma_load_2d(ring + size_t(st) * stage_bytes(p.regime), map, 0, static_cast<int32_t>(row), &full[st]);
     ++j;
   };
   if (p.regime == 0) {
@@ -347,8 +374,13 @@ __device__ void produce(const CUtensorMap* map, const Params& p, int64_t t_begin
         issue(t * p.step_rows + r0);
       }
   }
-  for (uint32_t i = j > uint32_t(kStages) ? j - kStages : 0; i < j; ++i)
-    drain_wait(&full[i % kStages], (i / kStages) & 1u);
+  // copies still in flight: at most one per stage, the last tiles issued
+  const uint32_t nst = p.regime == 0 ? kR0Stages : kR1Stages;
+  for (uint32_t i = j > nst ? j - nst : 0; i < j; ++i) {
+    uint32_t st, ph;
+    stage_of(p.regime, i, st, ph);
+    drain_wait(&full[st], ph);
+  }
 }
 
 // --------------------------------------------------------------------------
@@ -360,19 +392,19 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
   constexpr int NV = GAIN ? 2 * S : S;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* ring = align_1024(smem_raw);
-  uint64_t* full = reinterpret_cast<uint64_t*>(ring + size_t(kStages) * kTileBytes);
-  uint64_t* empty = full + kStages;
-  volatile int* abort = reinterpret_cast<volatile int*>(empty + kStages);
-  uint64_t* red = reinterpret_cast<uint64_t*>(empty + kStages) + 2;
+  uint64_t* full = reinterpret_cast<uint64_t*>(ring + kRingBytes);
+  uint64_t* empty = full + kMaxStages;
+  volatile int* abort = reinterpret_cast<volatile int*>(empty + kMaxStages);
+  uint64_t* red = reinterpret_cast<uint64_t*>(empty + kMaxStages) + 2;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t G = gridDim.x, b = blockIdx.x;
   const int64_t t_begin = p.T * b / G, t_end = p.T * (b + 1) / G;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < kStages; ++i) {
+    for (int i = 0; i < kMaxStages; ++i) {
       mbar_init(&full[i], 1);
-      mbar_init(&empty[i], p.regime == 0 ? static_cast<uint32_t>(p.K) : uint32_t(kConsumerWarps));
+      mbar_init(&empty[i], p.regime == 0 ? 1u : uint32_t(kConsumerWarps));
     }
     *abort = 0;
     fence_barrier_init();
@@ -390,68 +422,69 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
   const int R = static_cast<int>(p.R);
 
   if (p.regime == 0) {
-    // ---- one step per warp, K steps per tile
+    // ---- each warp owns every 8th tile (K whole steps) and two ring stages
     const int64_t n_local = t_end - t_begin;
-    for (int64_t i = warp; i < n_local; i += kConsumerWarps) {
-      const uint32_t j = static_cast<uint32_t>(i / p.K);
-      const uint32_t st = j % kStages, ph = (j / kStages) & 1u;
+    const int64_t n_tiles = (n_local + p.K - 1) / p.K;
+    uint32_t i = 0;
+    for (int64_t j = warp; j < n_tiles; j += kConsumerWarps, ++i) {
+      const uint32_t st = 2u * warp + (i & 1u), ph = (i >> 1) & 1u;
       const bool have = mbar_wait_bounded(&full[st], ph, abort);
-      const int kk = static_cast<int>(i - int64_t(j) * p.K);
-      const unsigned char* tile = ring + size_t(st) * kTileBytes;
-      const int64_t t = t_begin + i;
-      const int64_t w = GAIN ? t / p.W : 0;
-      if (GAIN && p.quality) qual_window(p, qa, w, lane);
-      const int q0 = kk * R;
-      if constexpr (!GAIN) {
-        FrontierRows<S> rs;
-        rs.init();
-        if (have) {
-          for (int r0 = lane; r0 < R; r0 += 32 * U) {
-            int64_t v[U][S];
+      const unsigned char* tile = ring + size_t(st) * kR0StageBytes;
+      const int nsteps = static_cast<int>(min(int64_t(p.K), n_local - j * p.K));
+      for (int kk = 0; kk < nsteps; ++kk) {
+        const int64_t t = t_begin + j * p.K + kk;
+        const int64_t w = GAIN ? t / p.W : 0;
+        if (GAIN && p.quality) qual_window(p, qa, w, lane);
+        const int q0 = kk * R;
+        if constexpr (!GAIN) {
+          FrontierRows<S> rs;
+          rs.init();
+          if (have) {
+            for (int r0 = lane; r0 < R; r0 += 32 * U) {
+              int64_t v[U][S];
 #pragma unroll
-            for (int u = 0; u < U; ++u)
-              if (r0 + 32 * u < R) load_row<S, kSwz>(tile, q0 + r0 + 32 * u, v[u]);
+              for (int u = 0; u < U; ++u)
+                if (r0 + 32 * u < R) load_row<S, kSwz>(tile, q0 + r0 + 32 * u, v[u]);
 #pragma unroll
-            for (int u = 0; u < U; ++u)
-              if (r0 + 32 * u < R) rs.row(v[u], r0 + 32 * u, dor, tor);
+              for (int u = 0; u < U; ++u)
+                if (r0 + 32 * u < R) rs.row(v[u], r0 + 32 * u, dor, tor);
+            }
           }
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&empty[st]);
-        uint64_t mykey = 0;
+          uint64_t mykey = 0;
 #pragma unroll
-        for (int s = 0; s < S; ++s) {
-          const uint64_t km = warp_max_u64(rs.key(s));
-          if (lane == s) mykey = km;
-        }
-        finalize_frontier(p, S, t, mykey, lane, acc);
-      } else {
-        GainRows<S> rs;
-        rs.init();
-        if (have) {
-          for (int r = lane; r < R; r += 32) {
-            int64_t v[S], mr[S];
-            load_row<S, kSwz>(tile, q0 + r, v);
-            load_global_row<S>(p.m + (w * p.R + r) * S, mr);
-            const int64_t total = rs.row(v, mr, dor, tor);
-            if (p.quality)
-              qual_row(p, qa, t, r, total, p.other_stage >= 0 ? pick<S>(v, p.other_stage) : 0, dor);
+          for (int s = 0; s < S; ++s) {
+            const uint64_t km = warp_max_u64(rs.key(s));
+            if (lane == s) mykey = km;
           }
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&empty[st]);
-        int64_t myF = 0, myR = 0;
+          finalize_frontier(p, S, t, mykey, lane, acc);
+        } else {
+          GainRows<S> rs;
+          rs.init();
+          if (have) {
+            for (int r = lane; r < R; r += 32) {
+              int64_t v[S], mr[S];
+              load_row<S, kSwz>(tile, q0 + r, v);
+              load_global_row<S>(p.m + (w * p.R + r) * S, mr);
+              const int64_t total = rs.row(v, mr, dor, tor);
+              if (p.quality)
+                qual_row(p, qa, t, r, total, p.other_stage >= 0 ? pick<S>(v, p.other_stage) : 0, dor);
+            }
+          }
+          int64_t myF = 0, myR = 0;
 #pragma unroll
-        for (int s = 0; s < S; ++s) {
-          const uint64_t f = warp_max_u64(static_cast<uint64_t>(rs.bf[s]));
-          const uint64_t g = warp_max_u64(static_cast<uint64_t>(rs.bg[s]));
-          if (lane == s) {
-            myF = static_cast<int64_t>(f);
-            myR = static_cast<int64_t>(g);
+          for (int s = 0; s < S; ++s) {
+            const uint64_t f = warp_max_u64(static_cast<uint64_t>(rs.bf[s]));
+            const uint64_t g = warp_max_u64(static_cast<uint64_t>(rs.bg[s]));
+            if (lane == s) {
+              myF = static_cast<int64_t>(f);
+              myR = static_cast<int64_t>(g);
+            }
           }
+          finalize_gain(p, S, t, myF, myR, lane, acc);
         }
-        finalize_gain(p, S, t, myF, myR, lane, acc);
       }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[st]);
     }
   } else {
     // ---- one step per CTA, tiles_per_step tiles per step
@@ -465,9 +498,9 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
       GainRows<S> gr;
       if constexpr (GAIN) gr.init(); else fr.init();
       for (int k = 0; k < p.tiles_per_step; ++k, ++j) {
-        const uint32_t st = j % kStages, ph = (j / kStages) & 1u;
+        const uint32_t st = j % kR1Stages, ph = (j / kR1Stages) & 1u;
         const bool have = mbar_wait_bounded(&full[st], ph, abort);
-        const unsigned char* tile = ring + size_t(st) * kTileBytes;
+        const unsigned char* tile = ring + size_t(st) * kR1StageBytes;
         const int64_t row0 = min(int64_t(k) * p.box_rows, p.step_rows - p.box_rows);
         const int rank_tile0 = static_cast<int>(row0 * 16 / S);
         const int rank_fresh = static_cast<int>(int64_t(k) * p.box_rows * 16 / S);
@@ -707,9 +740,9 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
   const int sms = sm_count();
   if (fast) {
     p.step_rows = step_rows;
-    if (step_rows <= kMaxBoxRows / 2) {
+    if (step_rows <= kR0MaxRows) {
       p.regime = 0;
-      p.K = static_cast<int>(kMaxBoxRows / step_rows);
+      p.K = static_cast<int>(kR0MaxRows / step_rows);
       p.box_rows = static_cast<int>(p.K * step_rows);
       p.tiles_per_step = 0;
     } else {
@@ -717,11 +750,11 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
       // rows per rank-aligned block: a tile must hold whole rank rows
       const int64_t elems = 16 * j.S / std::gcd<int64_t>(16, j.S);  // lcm(16, S)
       const int64_t q = elems / 16;
-      int64_t n = (step_rows + kMaxBoxRows - 1) / kMaxBoxRows, br = 0;
+      int64_t n = (step_rows + kR1MaxRows - 1) / kR1MaxRows, br = 0;
       for (;; ++n) {
         br = (step_rows + n - 1) / n;
         br = (br + q - 1) / q * q;
-        if (br <= kMaxBoxRows) break;
+        if (br <= kR1MaxRows) break;
       }
       p.box_rows = static_cast<int>(br);
       p.tiles_per_step = static_cast<int>((step_rows + br - 1) / br);

@@ -47,8 +47,8 @@ def make(T, R, S, seed, kind):
     return x
 
 
-# (T, R, S): generic path; fast path one-step-per-warp (<= 16 KB steps);
-# fast path one-step-per-CTA with overlapped last tile.
+# (T, R, S): generic path; fast path with warp-owned tiles of whole steps
+# (<= 12 KB steps); fast path one-step-per-CTA with overlapped last tile.
 SHAPES = [
     (37, 3, 5), (20, 1, 1), (11, 7, 32), (9, 65, 3), (6, 5, 18),          # generic
     (1000, 8, 6), (301, 128, 8), (123, 64, 4), (77, 64, 16), (50, 2, 8),   # one step per warp
@@ -70,6 +70,38 @@ def test_frontier_parity(sf, T, R, S, kind):
     assert np.array_equal(host(f.a), o.a)
     assert np.array_equal(host(f.lead), o.lead)
     assert np.array_equal(host(f.makespan), o.makespan)
+
+
+# Long step ranges: every CTA streams many tiles, so every ring stage is reused
+# many times (both regimes, both passes).
+LONG = [(200000, 8, 6), (20000, 64, 4), (8000, 128, 8), (3000, 512, 4), (1500, 1024, 10),
+        (600, 4096, 8)]
+
+
+@pytest.mark.parametrize("T,R,S", LONG)
+def test_long_ranges_reuse_ring(sf, T, R, S):
+    d_np = make(T, R, S, T + R, "ties" if R <= 64 else "lognormal")
+    W = 100
+    o = O.frontier(d_np)
+    ow = O.windows(d_np, W)
+    st = sf.new_status("cuda")
+    d = dev(d_np)
+    f = sf.sf_frontier(d, status=st)
+    g = sf.sf_window_aggregate(d, W, status=st)
+    m = sf.sf_window_median(d, W)
+    ev = sf.sf_direct_gain(d, W, m, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert np.array_equal(host(f.a), o.a) and np.array_equal(host(f.lead), o.lead)
+    assert np.array_equal(host(f.makespan), o.makespan)
+    for name in ("X", "D", "E", "C", "step_lead"):
+        assert np.array_equal(host(getattr(g, name)), getattr(ow, name)), name
+    assert np.array_equal(host(ev.X), ow.X) and np.array_equal(host(ev.D), ow.D)
+    assert np.array_equal(host(ev.step_lead) & 31, ow.step_lead)
+    # gain numerators on the first two windows (the literal oracle is S x slower)
+    m2 = O.window_median(d_np[:2 * W], W)
+    assert np.array_equal(host(m)[:2], m2)
+    assert np.array_equal(host(ev.Y)[:2], O.direct_gain(d_np[:2 * W], W, m2))
 
 
 @pytest.mark.parametrize("T,R,S", SHAPES[:4] + SHAPES[5:9] + SHAPES[14:18])
