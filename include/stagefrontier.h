@@ -218,6 +218,44 @@ sf_status sf_label_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, in
                            uint32_t* amb_mask, double* share, double* gain, int64_t* X,
                            int64_t* Y, int64_t* D, uint32_t* status, cudaStream_t stream);
 
+/*
+ * sf_label_windows_noalloc - sf_label_windows for callers that cannot
+ * allocate device memory.  The paper has no counterpart; this is a
+ * deployment variant of the labeler above.  It exists because an always-on
+ * monitor runs inside someone else's training job: the framework's caching
+ * allocator owns the device memory there, and a cudaMalloc issued from the
+ * monitoring hook can block on or synchronize the device (stalling the very
+ * step it measures) and carve memory out of that pool; a side-car with a
+ * fixed memory budget may have no allocator to call at all.
+ *
+ * Scratch: one static device array of SF_STATIC_SCRATCH_BYTES (16 MiB) in
+ * this library, held by every GPU that loads the library until the process
+ * exits.  A problem whose sf_label_windows_workspace_size exceeds it returns
+ * SF_EWORKSPACE before anything is enqueued.  The call allocates nothing and
+ * frees nothing.
+ *
+ * Set-up: the first call on each device looks up the array's device address
+ * (cudaGetSymbolAddress) with that device current, and caches it; make that
+ * first call before any stream capture.
+ *
+ * Sharing: all calls on a device use the same array, and it keeps whatever
+ * the last call left there.  Each call zeroes the parts it accumulates into,
+ * so calls ordered on one stream are independent; calls that can overlap on
+ * the GPU (other streams without an ordering event, concurrent host threads)
+ * race on the array and corrupt each other's results.
+ *
+ * Arguments, outputs and errors are those of sf_label_windows, without the
+ * workspace pair.
+ */
+#define SF_STATIC_SCRATCH_BYTES (16u * 1024u * 1024u)
+
+sf_status sf_label_windows_noalloc(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W,
+                                   const int32_t* role, const int32_t* missing, const int64_t* wall,
+                                   int32_t other_stage, const sf_label_config* cfg, uint32_t* labels,
+                                   uint32_t* route_mask, uint32_t* amb_mask, double* share,
+                                   double* gain, int64_t* X, int64_t* Y, int64_t* D,
+                                   uint32_t* status, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -1,6 +1,6 @@
 """Build libstagefrontier.so in-tree for sm_103a (nvcc, no cmake).
 
-The three translation units compile in parallel, then link into one shared
+The translation units compile in parallel, then link into one shared
 library with the CUDA runtime linked statically, so the library only talks to
 the driver through the handles (streams, device pointers) its caller passes.
 """
@@ -17,7 +17,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libstagefrontier.so")
-SOURCES = ["sf_stream.cu", "sf_select.cu", "sf_api.cu"]
+SOURCES = ["sf_stream.cu", "sf_select.cu", "sf_api.cu", "sf_static.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

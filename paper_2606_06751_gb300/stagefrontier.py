@@ -59,6 +59,8 @@ def _load():
                            P, P, P, S],
         "sf_label_windows": [P, I, I, I, I, P, P, P, I32, ctypes.POINTER(LabelConfig), P,
                              ctypes.c_size_t, P, P, P, P, P, P, P, P, P, S],
+        "sf_label_windows_noalloc": [P, I, I, I, I, P, P, P, I32, ctypes.POINTER(LabelConfig), P, P, P,
+                                     P, P, P, P, P, P, S],
     }
     for name, argt in sigs.items():
         f = getattr(L, name)
@@ -291,4 +293,23 @@ def sf_label_windows(d, W: int, role=None, missing=None, wall=None, other_stage:
                                  _p(out.route_mask), _p(out.amb_mask), _p(out.share), _p(out.gain),
                                  _p(out.X), _p(out.Y), _p(out.D), _p(status), _stream(stream)),
            "sf_label_windows")
+    return out
+
+
+STATIC_SCRATCH_BYTES = 16 * 1024 * 1024
+
+
+def sf_label_windows_noalloc(d, W: int, role=None, missing=None, wall=None, other_stage: int = -1,
+                             cfg=None, out: Labels = None, status=None, stream=None):
+    """The labeler with its intermediates in the library's static device
+    scratch (no workspace; the outputs are still the caller's tensors)."""
+    T, R, S = _d3(d)
+    cfg = cfg if cfg is not None else default_config()
+    if out is None:
+        raise ValueError("pass preallocated outputs (Labels with X, Y, D) to the no-allocation entry point")
+    _check(_lib.sf_label_windows_noalloc(_p(d), T, R, S, W, _p(role), _p(missing), _p(wall), other_stage,
+                                         ctypes.byref(cfg), _p(out.labels), _p(out.route_mask),
+                                         _p(out.amb_mask), _p(out.share), _p(out.gain), _p(out.X),
+                                         _p(out.Y), _p(out.D), _p(status), _stream(stream)),
+           "sf_label_windows_noalloc")
     return out
