@@ -303,7 +303,9 @@ def run_ours(args):
     for ev in timed:
         for i, n in enumerate(pipe.names):
             per_kernel[n].append(ev[i].elapsed_time(ev[i + 1]) / 1e3)
-    avg = {n: sum(v) / len(v) for n, v in per_kernel.items()}
+    # median over the timed steps: robust to the first step, which follows a
+    # synchronize and so also carries the host's enqueue latency
+    avg = {n: statistics.median(v) for n, v in per_kernel.items()}
     algo = pipe.algorithmic_bytes()
     dominant = max(avg, key=avg.get)
     peak, peak_kind = peaks()

@@ -25,46 +25,120 @@ __global__ void zero_kernel(uint32_t* __restrict__ p, size_t words) {
 // Lower median, one warp per column.  A CTA of 8 warps owns (window w, eight
 // consecutive flat columns c = r*S + s).  The window's rows of those columns
 // are read coalesced and transposed through shared memory so each warp holds
-// its column in registers (NPL values per lane).  Selection is a bitwise
-// search on the offset from the column minimum: the k-th smallest value
-// (k = floor((n-1)/2)) is the largest v with #{x < v} <= k, found one bit at
-// a time from the top bit of (max - min), each bit costing one warp-wide
-// count.  Values are compared as signed int64 (mapped to an order-preserving
-// unsigned key), so the result is exact for any input.
+// its column in registers (NPL values per lane).  Values are mapped to an
+// order-preserving unsigned key (so any int64 input is handled exactly) and
+// offset by the column minimum; the k-th smallest offset (k = floor((n-1)/2))
+// is then found by radix selection, most significant 8-bit digit first: a
+// per-warp 256-bin shared-memory histogram of the digit among the values that
+// share the digits chosen so far, a warp scan to find the bin holding rank k,
+// and the rank re-based into that bin.  A 24-bit spread takes three passes.
 constexpr int kMedCols = 8;
 constexpr int kMedThreads = kMedCols * 32;
+constexpr int kMedBins = 256;
 
-template <int NPL>
+// k-th smallest (0-based) of the lane-strided values x[i] (row lane + 32 i,
+// valid while row < n), all below 2^nbits.  hist: this warp's 256 counters.
+template <typename U, int NPL>
+__device__ __forceinline__ U warp_radix_select(const U (&x)[NPL], int n, int nbits, uint32_t k,
+                                               uint32_t* hist, int lane) {
+  U prefix = 0;
+  int shift = nbits;
+  uint32_t rem = k;
+  bool first = true;
+  while (shift > 0) {
+    const int D = shift < 8 ? shift : 8;
+    shift -= D;
+    const uint32_t dmask = (1u << D) - 1u;
+    const int hs = shift + D;  // bits above the current digit
+    reinterpret_cast<uint4*>(hist)[2 * lane] = make_uint4(0, 0, 0, 0);
+    reinterpret_cast<uint4*>(hist)[2 * lane + 1] = make_uint4(0, 0, 0, 0);
+    __syncwarp();
+#pragma unroll
+    for (int i = 0; i < NPL; ++i) {
+      if (lane + 32 * i < n) {
+        const U v = x[i];
+        if (first || (v >> hs) == prefix)
+          atomicAdd(&hist[static_cast<uint32_t>(v >> shift) & dmask], 1u);
+      }
+    }
+    __syncwarp();
+    const uint4 h0 = reinterpret_cast<const uint4*>(hist)[2 * lane];
+    const uint4 h1 = reinterpret_cast<const uint4*>(hist)[2 * lane + 1];
+    const uint32_t hb[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+    uint32_t sum = 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) sum += hb[j];
+    uint32_t incl = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t up = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += up;
+    }
+    const uint32_t excl = incl - sum;
+    const int owner = __ffs(__ballot_sync(kFull, excl <= rem && rem < incl)) - 1;
+    uint32_t digit = 0, below = excl;
+    if (lane == owner) {
+      uint32_t c = excl;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        if (rem >= c && rem < c + hb[j]) {
+          digit = 8u * lane + j;
+          below = c;
+        }
+        c += hb[j];
+      }
+    }
+    digit = __shfl_sync(kFull, digit, owner);
+    below = __shfl_sync(kFull, below, owner);
+    rem -= below;
+    prefix = (prefix << D) | static_cast<U>(digit);
+    first = false;
+    __syncwarp();
+  }
+  return prefix;
+}
+
+template <int NPL, bool kVec>
 __global__ void __launch_bounds__(kMedThreads)
     median_kernel(const int64_t* __restrict__ d, int64_t T, int64_t RS, int64_t W, int64_t ngroups,
                   int64_t* __restrict__ m) {
   constexpr int LD = 32 * NPL + 1;
-  extern __shared__ int64_t colbuf[];  // [kMedCols][LD]
+  extern __shared__ int64_t colbuf[];  // [kMedCols][LD], then kMedCols x 256 histogram counters
+  // kMedCols * LD * 8 bytes is a multiple of 64, so the counters start 16-byte aligned
+  uint32_t* hists = reinterpret_cast<uint32_t*>(colbuf + kMedCols * LD);
   const int64_t w = blockIdx.x / ngroups;
   const int64_t c0 = (blockIdx.x % ngroups) * kMedCols;
   const int ncols = static_cast<int>(imin64(kMedCols, RS - c0));
   const int64_t tb = w * W;
   const int n = static_cast<int>(imin64(W, T - tb));
   const int64_t* base = d + tb * RS + c0;
-  for (int idx = threadIdx.x; idx < n * kMedCols; idx += kMedThreads) {
-    const int row = idx / kMedCols, c = idx % kMedCols;
-    colbuf[c * LD + row] = c < ncols ? __ldg(base + int64_t(row) * RS + c) : 0;
+  if (kVec && ncols == kMedCols) {  // 16-byte loads of column pairs (RS even)
+    for (int idx = threadIdx.x; idx < n * (kMedCols / 2); idx += kMedThreads) {
+      const int row = idx / (kMedCols / 2), pr = idx % (kMedCols / 2);
+      const longlong2 v = __ldg(reinterpret_cast<const longlong2*>(base + int64_t(row) * RS) + pr);
+      colbuf[(2 * pr) * LD + row] = v.x;
+      colbuf[(2 * pr + 1) * LD + row] = v.y;
+    }
+  } else {
+    for (int idx = threadIdx.x; idx < n * kMedCols; idx += kMedThreads) {
+      const int row = idx / kMedCols, c = idx % kMedCols;
+      colbuf[c * LD + row] = c < ncols ? __ldg(base + int64_t(row) * RS + c) : 0;
+    }
   }
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (warp >= ncols) return;
+  uint32_t* hist = hists + warp * kMedBins;  // 1 KB per warp
   constexpr uint64_t kSign = 1ull << 63;
   uint64_t u[NPL];
   uint64_t lo = ~0ull, hi = 0;
 #pragma unroll
   for (int i = 0; i < NPL; ++i) {
     const int row = lane + 32 * i;
+    u[i] = row < n ? static_cast<uint64_t>(colbuf[warp * LD + row]) ^ kSign : 0;
     if (row < n) {
-      u[i] = static_cast<uint64_t>(colbuf[warp * LD + row]) ^ kSign;
       lo = u[i] < lo ? u[i] : lo;
       hi = u[i] > hi ? u[i] : hi;
-    } else {
-      u[i] = ~0ull;  // padding sorts after every real value
     }
   }
   lo = warp_min_u64(lo);
@@ -72,33 +146,16 @@ __global__ void __launch_bounds__(kMedThreads)
   const uint32_t k = static_cast<uint32_t>((n - 1) / 2);
   const uint64_t range = hi - lo;
   const int nbits = range ? 64 - __clzll(static_cast<long long>(range)) : 0;
-  uint64_t ans = 0;
+  uint64_t ans;
   if (nbits <= 32) {
     uint32_t x[NPL];
 #pragma unroll
-    for (int i = 0; i < NPL; ++i) {
-      const uint64_t off = u[i] - lo;
-      x[i] = off > 0xffffffffull ? 0xffffffffu : static_cast<uint32_t>(off);
-    }
-    uint32_t a32 = 0;
-    for (int bit = nbits - 1; bit >= 0; --bit) {
-      const uint32_t cand = a32 | (1u << bit);
-      uint32_t cnt = 0;
-#pragma unroll
-      for (int i = 0; i < NPL; ++i) cnt += x[i] < cand ? 1u : 0u;
-      cnt = __reduce_add_sync(kFull, cnt);
-      if (cnt <= k) a32 = cand;
-    }
-    ans = a32;
+    for (int i = 0; i < NPL; ++i) x[i] = static_cast<uint32_t>(u[i] - lo);  // padding rows never read
+    ans = warp_radix_select<uint32_t, NPL>(x, n, nbits, k, hist, lane);
   } else {
-    for (int bit = nbits - 1; bit >= 0; --bit) {
-      const uint64_t cand = ans | (1ull << bit);
-      uint32_t cnt = 0;
 #pragma unroll
-      for (int i = 0; i < NPL; ++i) cnt += (u[i] - lo) < cand ? 1u : 0u;
-      cnt = __reduce_add_sync(kFull, cnt);
-      if (cnt <= k) ans = cand;
-    }
+    for (int i = 0; i < NPL; ++i) u[i] -= lo;
+    ans = warp_radix_select<uint64_t, NPL>(u, n, nbits, k, hist, lane);
   }
   if (lane == 0) m[w * RS + c0 + warp] = static_cast<int64_t>((lo + ans) ^ kSign);
 }
@@ -354,11 +411,13 @@ __global__ void __launch_bounds__(kGateThreads) gates_kernel(const GateJob g) {
 template <int NPL>
 cudaError_t launch_median_npl(const int64_t* d, int64_t T, int64_t RS, int64_t W, int64_t nW,
                               int64_t ngroups, int64_t* m, cudaStream_t stream) {
-  const size_t smem = size_t(kMedCols) * (32 * NPL + 1) * sizeof(int64_t);
-  cudaError_t e = cudaFuncSetAttribute(median_kernel<NPL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
+  const size_t smem = size_t(kMedCols) * (32 * NPL + 1) * sizeof(int64_t) +
+                      size_t(kMedCols) * kMedBins * sizeof(uint32_t);
+  const bool vec = (RS % 2) == 0 && (reinterpret_cast<uintptr_t>(d) % 16) == 0;
+  auto kern = vec ? median_kernel<NPL, true> : median_kernel<NPL, false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  median_kernel<NPL><<<static_cast<unsigned>(nW * ngroups), kMedThreads, smem, stream>>>(d, T, RS, W, ngroups, m);
+  kern<<<static_cast<unsigned>(nW * ngroups), kMedThreads, smem, stream>>>(d, T, RS, W, ngroups, m);
   return cudaGetLastError();
 }
 

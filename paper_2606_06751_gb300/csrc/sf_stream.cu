@@ -47,6 +47,9 @@ constexpr int kR0MaxRows = kR0StageBytes / kRowBytes;   // 96 rows
 constexpr int kR1Stages = 6;
 constexpr int kR1StageBytes = kRingBytes / kR1Stages;  // 32 KB
 constexpr int kR1MaxRows = kR1StageBytes / kRowBytes;   // 256 rows (the TMA box limit)
+// The evidence pass streams the window medians m next to d: each 32 KB stage
+// holds a d tile in its first half and the matching m tile in its second.
+constexpr int kR1GainMaxRows = kR1MaxRows / 2;
 constexpr int kMaxStages = kR0Stages;
 constexpr int kRedSlots = 2 * kConsumerWarps * 32;    // double-buffered per-warp partials
 constexpr size_t kSmemBytes = 1024 /*alignment slack*/ + size_t(kRingBytes) +
@@ -73,6 +76,7 @@ struct Params {
   int64_t* Y;
   uint64_t* quality;
   uint32_t* status;
+  int m_by_tma;  // evidence pass, regime 1: m tiles arrive through the ring
 };
 
 __device__ __forceinline__ uint32_t hi32(int64_t v) {
@@ -348,30 +352,34 @@ __device__ __forceinline__ size_t stage_bytes(int regime) {
   return regime == 0 ? size_t(kR0StageBytes) : size_t(kR1StageBytes);
 }
 
-__device__ void produce(const CUtensorMap* map, const Params& p, int64_t t_begin, int64_t t_end,
-                        unsigned char* ring, uint64_t* full, uint64_t* empty, volatile int* abort) {
+__device__ void produce(const CUtensorMap* map, const CUtensorMap* map_m, const Params& p, int64_t t_begin,
+                        int64_t t_end, unsigned char* ring, uint64_t* full, uint64_t* empty,
+                        volatile int* abort) {
   prefetch_tensormap(map);
+  if (p.m_by_tma) prefetch_tensormap(map_m);
   const uint32_t bytes = static_cast<uint32_t>(p.box_rows) * kRowBytes;
   uint32_t j = 0;  // tiles issued
   bool ok = true;
-  auto issue = [&](int64_t row) {
+  auto issue = [&](int64_t row, int64_t mrow) {
     uint32_t st, ph;
     stage_of(p.regime, j, st, ph);
     if (!mbar_wait_bounded(&empty[st], ph ^ 1u, abort)) {
       ok = false;
       return;
     }
-    mbar_arrive_expect_tx(&full[st], bytes);
-    tma_load_2d(ring + size_t(st) * stage_bytes(p.regime), map, 0, static_cast<int32_t>(row), &full[st]);
+    unsigned char* dst = ring + size_t(st) * stage_bytes(p.regime);
+    mbar_arrive_expect_tx(&full[st], p.m_by_tma ? 2u * bytes : bytes);
+    tma_load_2d(dst, map, 0, static_cast<int32_t>(row), &full[st]);
+    if (p.m_by_tma) tma_load_2d(dst + kR1StageBytes / 2, map_m, 0, static_cast<int32_t>(mrow), &full[st]);
     ++j;
   };
   if (p.regime == 0) {
-    for (int64_t t = t_begin; t < t_end && ok; t += p.K) issue(t * p.step_rows);
+    for (int64_t t = t_begin; t < t_end && ok; t += p.K) issue(t * p.step_rows, 0);
   } else {
     for (int64_t t = t_begin; t < t_end && ok; ++t)
       for (int k = 0; k < p.tiles_per_step && ok; ++k) {
         const int64_t r0 = min(int64_t(k) * p.box_rows, p.step_rows - p.box_rows);
-        issue(t * p.step_rows + r0);
+        issue(t * p.step_rows + r0, (t / p.W) * p.step_rows + r0);
       }
   }
   // copies still in flight: at most one per stage, the last tiles issued
@@ -386,7 +394,8 @@ __device__ void produce(const CUtensorMap* map, const Params& p, int64_t t_begin
 // --------------------------------------------------------------------------
 template <int S, bool GAIN>
 __global__ void __launch_bounds__(kBlockThreads, 1)
-    stream_kernel(const __grid_constant__ CUtensorMap map, const Params p) {
+    stream_kernel(const __grid_constant__ CUtensorMap map, const __grid_constant__ CUtensorMap map_m,
+                  const Params p) {
   constexpr bool kSwz = (S == 4 || S == 8 || S == 16);
   constexpr int U = S <= 8 ? 4 : 2;  // rank rows in flight per thread
   constexpr int NV = GAIN ? 2 * S : S;
@@ -412,7 +421,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
   __syncthreads();
 
   if (warp == kConsumerWarps) {
-    if (lane == 0) produce(&map, p, t_begin, t_end, ring, full, empty, abort);
+    if (lane == 0) produce(&map, &map_m, p, t_begin, t_end, ring, full, empty, abort);
     return;
   }
 
@@ -521,7 +530,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
             for (int r = rank_fresh + ctid; r < rank_end; r += kConsumerThreads) {
               int64_t v[S], mr[S];
               load_row<S, kSwz>(tile, r - rank_tile0, v);
-              load_global_row<S>(p.m + (w * p.R + r) * S, mr);
+              load_row<S, kSwz>(tile + kR1StageBytes / 2, r - rank_tile0, mr);  // m tile of the same ranks
               const int64_t total = gr.row(v, mr, dor, tor);
               if (p.quality)
                 qual_row(p, qa, t, r, total, p.other_stage >= 0 ? pick<S>(v, p.other_stage) : 0, dor);
@@ -680,12 +689,13 @@ cudaError_t prepare_fast() {
 }
 
 template <bool GAIN>
-cudaError_t dispatch_fast(int S, const CUtensorMap& map, const Params& p, int grid, cudaStream_t stream) {
+cudaError_t dispatch_fast(int S, const CUtensorMap& map, const CUtensorMap& map_m, const Params& p, int grid,
+                          cudaStream_t stream) {
 #define SF_CASE(SV)                                                                          \
   case SV: {                                                                                 \
     cudaError_t e = prepare_fast<SV, GAIN>();                                     \
     if (e != cudaSuccess) return e;                                                          \
-    stream_kernel<SV, GAIN><<<grid, kBlockThreads, kSmemBytes, stream>>>(map, p);            \
+    stream_kernel<SV, GAIN><<<grid, kBlockThreads, kSmemBytes, stream>>>(map, map_m, p);     \
     return cudaGetLastError();                                                               \
   }
   switch (S) {
@@ -750,32 +760,42 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
       // rows per rank-aligned block: a tile must hold whole rank rows
       const int64_t elems = 16 * j.S / std::gcd<int64_t>(16, j.S);  // lcm(16, S)
       const int64_t q = elems / 16;
-      int64_t n = (step_rows + kR1MaxRows - 1) / kR1MaxRows, br = 0;
+      const int64_t max_rows = j.gain ? kR1GainMaxRows : kR1MaxRows;
+      int64_t n = (step_rows + max_rows - 1) / max_rows, br = 0;
       for (;; ++n) {
         br = (step_rows + n - 1) / n;
         br = (br + q - 1) / q * q;
-        if (br <= kR1MaxRows) break;
+        if (br <= max_rows) break;
       }
       p.box_rows = static_cast<int>(br);
       p.tiles_per_step = static_cast<int>((step_rows + br - 1) / br);
       p.K = 0;
     }
-    CUtensorMap map;
-    const cuuint64_t gdim[2] = {16, static_cast<cuuint64_t>(rows_total)};
-    const cuuint64_t gstride[1] = {kRowBytes};
-    const cuuint32_t box[2] = {16, static_cast<cuuint32_t>(p.box_rows)};
-    const cuuint32_t estride[2] = {1, 1};
     const bool swz = (j.S == 4 || j.S == 8 || j.S == 16);
-    CUresult cr = encode_fn()(&map, CU_TENSOR_MAP_DATA_TYPE_INT64, 2, const_cast<int64_t*>(j.d), gdim,
-                              gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                              swz ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
-                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    auto encode = [&](CUtensorMap* out, const int64_t* base, int64_t rows) {
+      const cuuint64_t gdim[2] = {16, static_cast<cuuint64_t>(rows)};
+      const cuuint64_t gstride[1] = {kRowBytes};
+      const cuuint32_t box[2] = {16, static_cast<cuuint32_t>(p.box_rows)};
+      const cuuint32_t estride[2] = {1, 1};
+      return encode_fn()(out, CU_TENSOR_MAP_DATA_TYPE_INT64, 2, const_cast<int64_t*>(base), gdim, gstride, box,
+                         estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                         swz ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    };
+    CUtensorMap map, map_m;
+    if (encode(&map, j.d, rows_total) != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    map_m = map;
+    p.m_by_tma = (j.gain && p.regime == 1) ? 1 : 0;
+    if (p.m_by_tma) {
+      const int64_t nW = (j.T + j.W - 1) / j.W;
+      if (nW * step_rows > int64_t(0x7fffffff) || encode(&map_m, j.m, nW * step_rows) != CUDA_SUCCESS)
+        return cudaErrorInvalidValue;
+    }
     const int64_t units = p.regime == 0 ? (j.T + p.K - 1) / p.K : j.T;
     const int grid = static_cast<int>(std::min<int64_t>(sms, units));
     count_launch();
-    return j.gain ? dispatch_fast<true>(static_cast<int>(j.S), map, p, grid, stream)
-                  : dispatch_fast<false>(static_cast<int>(j.S), map, p, grid, stream);
+    return j.gain ? dispatch_fast<true>(static_cast<int>(j.S), map, map_m, p, grid, stream)
+                  : dispatch_fast<false>(static_cast<int>(j.S), map, map_m, p, grid, stream);
   }
   const int grid = static_cast<int>(std::min<int64_t>(int64_t(sms) * 4, j.T));
   count_launch();
