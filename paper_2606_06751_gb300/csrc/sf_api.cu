@@ -182,12 +182,12 @@ sf_status sf_topk_suspects(const int64_t* X, const int64_t* E, int64_t nW, int64
 
 sf_status sf_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W, int64_t* m,
                            uint32_t* status, cudaStream_t stream) {
-  (void)status;  // the median is defined for every int64 input
+  // the median is defined for every int64 input; status only reports a bounded wait that ran out
   if (!d || !m || !shape_ok(T, R, S) || W < 1 || W > 65536) return SF_EINVAL;
-  if (!aligned(d, 16) || !aligned(m, 8)) return SF_EINVAL_ALIGN;
+  if (!aligned(d, 16) || !aligned(m, 8) || !aligned(status, 4)) return SF_EINVAL_ALIGN;
   const int64_t nW = (T + W - 1) / W;
   if (nW * ((R * S + 7) / 8) > 0x7fffffff) return SF_EUNSUPPORTED;
-  return cuda_status(launch_window_median(d, T, R, S, W, m, stream));
+  return cuda_status(launch_window_median(d, T, R, S, W, m, status, stream));
 }
 
 sf_status sf_direct_gain(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W, const int64_t* m,

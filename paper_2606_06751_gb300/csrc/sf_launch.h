@@ -2,6 +2,7 @@
 // the kernel translation units.  Internal to libstagefrontier.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -35,13 +36,20 @@ struct StreamJob {
   uint32_t* status = nullptr;
 };
 
+// cuTensorMapEncodeTiled from the driver, resolved once (null if unavailable).
+using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                              const cuuint64_t*, const cuuint32_t*, const cuuint32_t*,
+                              CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                              CUtensorMapFloatOOBfill);
+EncodeFn encode_fn();
+
 int sm_count();                     // SMs of the current device (cached)
 void count_launch(uint64_t n = 1);  // bump the library's launch counter
 
 cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t stream);
 cudaError_t launch_stream_pass(const StreamJob& job, cudaStream_t stream);
 cudaError_t launch_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W,
-                                 int64_t* m, cudaStream_t stream);
+                                 int64_t* m, uint32_t* status, cudaStream_t stream);
 cudaError_t launch_topk(const int64_t* X, const int64_t* E, int64_t nW, int64_t S, int64_t R,
                         int32_t k, int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair,
                         int64_t* top_pair_value, cudaStream_t stream);

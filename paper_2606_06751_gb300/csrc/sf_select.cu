@@ -36,11 +36,11 @@ constexpr int kMedCols = 8;
 constexpr int kMedThreads = kMedCols * 32;
 constexpr int kMedBins = 256;
 
-// k-th smallest (0-based) of the lane-strided values x[i] (row lane + 32 i,
+// k-th smallest (0-based) of the lane-strided values get(i) (row lane + 32 i,
 // valid while row < n), all below 2^nbits.  hist: this warp's 256 counters.
-template <typename U, int NPL>
-__device__ __forceinline__ U warp_radix_select(const U (&x)[NPL], int n, int nbits, uint32_t k,
-                                               uint32_t* hist, int lane) {
+template <typename U, int NPL, typename Get>
+__device__ __forceinline__ U warp_radix_select(Get get, int n, int nbits, uint32_t k, uint32_t* hist,
+                                               int lane) {
   U prefix = 0;
   int shift = nbits;
   uint32_t rem = k;
@@ -56,7 +56,7 @@ __device__ __forceinline__ U warp_radix_select(const U (&x)[NPL], int n, int nbi
 #pragma unroll
     for (int i = 0; i < NPL; ++i) {
       if (lane + 32 * i < n) {
-        const U v = x[i];
+        const U v = get(i);
         if (first || (v >> hs) == prefix)
           atomicAdd(&hist[static_cast<uint32_t>(v >> shift) & dmask], 1u);
       }
@@ -151,11 +151,95 @@ __global__ void __launch_bounds__(kMedThreads)
     uint32_t x[NPL];
 #pragma unroll
     for (int i = 0; i < NPL; ++i) x[i] = static_cast<uint32_t>(u[i] - lo);  // padding rows never read
-    ans = warp_radix_select<uint32_t, NPL>(x, n, nbits, k, hist, lane);
+    ans = warp_radix_select<uint32_t, NPL>([&](int i) { return x[i]; }, n, nbits, k, hist, lane);
   } else {
 #pragma unroll
     for (int i = 0; i < NPL; ++i) u[i] -= lo;
-    ans = warp_radix_select<uint64_t, NPL>(u, n, nbits, k, hist, lane);
+    ans = warp_radix_select<uint64_t, NPL>([&](int i) { return u[i]; }, n, nbits, k, hist, lane);
+  }
+  if (lane == 0) m[w * RS + c0 + warp] = static_cast<int64_t>((lo + ans) ^ kSign);
+}
+
+// The same selection with the window tile brought in by bulk tensor copies: one
+// thread issues the whole (window x 8 columns) tile, up to four 2-D boxes of
+// 8 int64 x box_rows, all completing on one mbarrier.  The tile stays row-major
+// (64-byte rows) with the 64-byte swizzle, so a warp reading one column down
+// 32 rows touches 8 distinct 16-byte bank groups per 16 lanes.  Offsets from
+// the column minimum stay in registers only when they fit 32 bits; wider
+// columns re-read shared memory on every radix pass.  Registers are capped so
+// three CTAs share an SM and one CTA's copy overlaps another's selection.
+__device__ __forceinline__ int64_t tile_at(const unsigned char* tile, int r, int c) {
+  const uint32_t off = uint32_t(r) * 64u + ((uint32_t(c >> 1) ^ ((uint32_t(r) >> 1) & 3u)) << 4) + (uint32_t(c & 1) << 3);
+  return *reinterpret_cast<const int64_t*>(tile + off);
+}
+
+template <int NPL>
+__global__ void __launch_bounds__(kMedThreads, 3)
+    median_tma_kernel(const __grid_constant__ CUtensorMap map, int64_t T, int64_t RS, int64_t W,
+                      int64_t ngroups, int box_rows, int nbox, int64_t* __restrict__ m, uint32_t* status) {
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* tile = align_1024(smem_raw);
+  const uint32_t tile_bytes = uint32_t(nbox) * uint32_t(box_rows) * 64u;
+  uint32_t* hists = reinterpret_cast<uint32_t*>(tile + tile_bytes);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(hists + kMedCols * kMedBins);
+  volatile int* abort = reinterpret_cast<volatile int*>(bar + 1);
+  const int64_t w = blockIdx.x / ngroups;
+  const int64_t c0 = (blockIdx.x % ngroups) * kMedCols;
+  const int ncols = static_cast<int>(imin64(kMedCols, RS - c0));
+  const int64_t tb = w * W;
+  const int n = static_cast<int>(imin64(W, T - tb));
+  if (threadIdx.x == 0) {
+    mbar_init(bar, 1);
+    *abort = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    mbar_arrive_expect_tx(bar, tile_bytes);
+    for (int b = 0; b < nbox; ++b)
+      tma_load_2d(tile + size_t(b) * box_rows * 64, &map, static_cast<int32_t>(c0),
+                  static_cast<int32_t>(tb + int64_t(b) * box_rows), bar);
+  }
+  const bool ok = mbar_wait_bounded(bar, 0, abort);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (!ok) {
+    if (threadIdx.x == 0) {
+      report(status, SF_ST_TIMEOUT);
+      mbar_wait_timeout(bar, 0);  // let the copies land before the CTA's memory is released
+    }
+    return;
+  }
+  if (warp >= ncols) return;
+  uint32_t* hist = hists + warp * kMedBins;
+  constexpr uint64_t kSign = 1ull << 63;
+  uint64_t lo = ~0ull, hi = 0;
+#pragma unroll
+  for (int i = 0; i < NPL; ++i) {
+    const int row = lane + 32 * i;
+    if (row < n) {
+      const uint64_t u = static_cast<uint64_t>(tile_at(tile, row, warp)) ^ kSign;
+      lo = u < lo ? u : lo;
+      hi = u > hi ? u : hi;
+    }
+  }
+  lo = warp_min_u64(lo);
+  hi = warp_max_u64(hi);
+  const uint32_t k = static_cast<uint32_t>((n - 1) / 2);
+  const uint64_t range = hi - lo;
+  const int nbits = range ? 64 - __clzll(static_cast<long long>(range)) : 0;
+  uint64_t ans;
+  if (nbits <= 32) {
+    uint32_t x[NPL];
+#pragma unroll
+    for (int i = 0; i < NPL; ++i) {
+      const int row = lane + 32 * i;
+      x[i] = row < n ? static_cast<uint32_t>((static_cast<uint64_t>(tile_at(tile, row, warp)) ^ kSign) - lo) : 0u;
+    }
+    ans = warp_radix_select<uint32_t, NPL>([&](int i) { return x[i]; }, n, nbits, k, hist, lane);
+  } else {
+    ans = warp_radix_select<uint64_t, NPL>(
+        [&](int i) { return (static_cast<uint64_t>(tile_at(tile, lane + 32 * i, warp)) ^ kSign) - lo; }, n, nbits,
+        k, hist, lane);
   }
   if (lane == 0) m[w * RS + c0 + warp] = static_cast<int64_t>((lo + ans) ^ kSign);
 }
@@ -421,6 +505,19 @@ cudaError_t launch_median_npl(const int64_t* d, int64_t T, int64_t RS, int64_t W
   return cudaGetLastError();
 }
 
+template <int NPL>
+cudaError_t launch_median_tma(const CUtensorMap& map, int64_t T, int64_t RS, int64_t W, int64_t nW,
+                              int64_t ngroups, int box_rows, int nbox, int64_t* m, uint32_t* status,
+                              cudaStream_t stream) {
+  const size_t smem = 1024 + size_t(nbox) * box_rows * 64 + size_t(kMedCols) * kMedBins * 4 + 16;
+  cudaError_t e =
+      cudaFuncSetAttribute(median_tma_kernel<NPL>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  median_tma_kernel<NPL><<<static_cast<unsigned>(nW * ngroups), kMedThreads, smem, stream>>>(
+      map, T, RS, W, ngroups, box_rows, nbox, m, status);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t stream) {
@@ -433,12 +530,34 @@ cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t stream) {
 }
 
 cudaError_t launch_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W,
-                                 int64_t* m, cudaStream_t stream) {
+                                 int64_t* m, uint32_t* status, cudaStream_t stream) {
   const int64_t RS = R * S;
   const int64_t nW = (T + W - 1) / W;
   const int64_t ngroups = (RS + kMedCols - 1) / kMedCols;
   const int64_t n = std::min(W, T);
   count_launch();
+  // Bulk-copy path: rows of d are 16-byte multiples (RS even), d is 16-byte
+  // aligned, windows fit the register path, the driver encoder is available.
+  if (RS % 2 == 0 && reinterpret_cast<uintptr_t>(d) % 16 == 0 && n <= 1024 && T < (int64_t(1) << 31) &&
+      encode_fn() != nullptr) {
+    const int nbox = static_cast<int>((n + 255) / 256);
+    const int box_rows = static_cast<int>(((n + nbox - 1) / nbox + 15) / 16 * 16);  // 1024-byte boxes
+    CUtensorMap map;
+    const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(RS), static_cast<cuuint64_t>(T)};
+    const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(RS) * 8};
+    const cuuint32_t box[2] = {static_cast<cuuint32_t>(kMedCols), static_cast<cuuint32_t>(box_rows)};
+    const cuuint32_t estride[2] = {1, 1};
+    if (encode_fn()(&map, CU_TENSOR_MAP_DATA_TYPE_INT64, 2, const_cast<int64_t*>(d), gdim, gstride, box, estride,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS) {
+      if (n <= 32) return launch_median_tma<1>(map, T, RS, W, nW, ngroups, box_rows, nbox, m, status, stream);
+      if (n <= 64) return launch_median_tma<2>(map, T, RS, W, nW, ngroups, box_rows, nbox, m, status, stream);
+      if (n <= 128) return launch_median_tma<4>(map, T, RS, W, nW, ngroups, box_rows, nbox, m, status, stream);
+      if (n <= 256) return launch_median_tma<8>(map, T, RS, W, nW, ngroups, box_rows, nbox, m, status, stream);
+      if (n <= 512) return launch_median_tma<16>(map, T, RS, W, nW, ngroups, box_rows, nbox, m, status, stream);
+      return launch_median_tma<32>(map, T, RS, W, nW, ngroups, box_rows, nbox, m, status, stream);
+    }
+  }
   if (n <= 32) return launch_median_npl<1>(d, T, RS, W, nW, ngroups, m, stream);
   if (n <= 64) return launch_median_npl<2>(d, T, RS, W, nW, ngroups, m, stream);
   if (n <= 128) return launch_median_npl<4>(d, T, RS, W, nW, ngroups, m, stream);

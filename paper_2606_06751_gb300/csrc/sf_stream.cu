@@ -321,20 +321,6 @@ __device__ __forceinline__ void load_global_row(const int64_t* src, int64_t (&v)
   }
 }
 
-// Offset the dynamic shared-memory base to the next 1024-byte boundary (the
-// 128-byte swizzle pattern repeats every 1024 bytes); pointer arithmetic keeps
-// the shared address space visible to the compiler.
-__device__ __forceinline__ unsigned char* align_1024(unsigned char* p) {
-  return p + ((1024u - (smem_u32(p) & 1023u)) & 1023u);
-}
-
-// Wait (bounded, ignoring abort) for copies still in flight before the CTA exits.
-__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
-  if (mbar_try_wait(bar, parity)) return;
-  const uint64_t t0 = global_timer_ns();
-  while (!mbar_try_wait(bar, parity))
-    if (global_timer_ns() - t0 > kWaitLimitNs) return;
-}
 
 // Ring stage and phase parity of the j-th tile a CTA streams.
 __device__ __forceinline__ void stage_of(int regime, uint32_t j, uint32_t& st, uint32_t& ph) {
@@ -387,7 +373,7 @@ __device__ void produce(const CUtensorMap* map, const CUtensorMap* map_m, const 
   for (uint32_t i = j > nst ? j - nst : 0; i < j; ++i) {
     uint32_t st, ph;
     stage_of(p.regime, i, st, ph);
-    drain_wait(&full[st], ph);
+    mbar_wait_timeout(&full[st], ph);
   }
 }
 
@@ -664,24 +650,6 @@ __global__ void __launch_bounds__(kGenThreads)
 
 // --------------------------------------------------------------------------
 // Host side
-using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                              const cuuint64_t*, const cuuint32_t*, const cuuint32_t*,
-                              CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
-                              CUtensorMapFloatOOBfill);
-
-EncodeFn encode_fn() {
-  static EncodeFn fn = [] {
-    void* f = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
-            cudaSuccess ||
-        q != cudaDriverEntryPointSuccess)
-      f = nullptr;
-    return reinterpret_cast<EncodeFn>(f);
-  }();
-  return fn;
-}
-
 template <int S, bool GAIN>
 cudaError_t prepare_fast() {
   return cudaFuncSetAttribute(stream_kernel<S, GAIN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -714,6 +682,19 @@ cudaError_t dispatch_fast(int S, const CUtensorMap& map, const CUtensorMap& map_
 }
 
 }  // namespace
+
+EncodeFn encode_fn() {
+  static EncodeFn fn = [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      f = nullptr;
+    return reinterpret_cast<EncodeFn>(f);
+  }();
+  return fn;
+}
 
 cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
   Params p{};
