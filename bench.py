@@ -3,7 +3,7 @@
 One step = one pass of the whole path over one batch of synthetic telemetry:
 window aggregation fused into the frontier pass (Sec. 3 Eq. 1-2), top-k
 suspects, and the labeler (per-rank window medians, the clipped-gain evidence
-pass of Sec. 4 Eq. 3, App. C gates).  The default workload is the largest
+pass of Sec. 4 Eq. 4, App. C gates).  The default workload is the largest
 frontier-accounting configuration: 8192 ranks x 8 stages x 20000 steps of
 int64 ns (10.49 GB), 1000-step windows, top-5, labels.
 

@@ -148,7 +148,7 @@ typedef struct sf_label_config {
 void sf_label_config_default(sf_label_config* cfg);
 
 /*
- * sf_window_median - the per-rank window baseline of Sec. 4 (Eq. 3): for each
+ * sf_window_median - the per-rank window baseline of Sec. 4 (Eq. 4): for each
  * window w (steps [wW, min((w+1)W, T)) of d, starting at d's first step), rank
  * r and stage s, the LOWER median of {d[t,r,s]}: element floor((n-1)/2) of the
  * ascending order, n the window's step count.
@@ -159,7 +159,7 @@ sf_status sf_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, in
 
 /*
  * sf_direct_gain - the evidence pass of the labeler (Sec. 4): per window the
- * Eq. 2 numerators X and denominator D, the Eq. 3 numerators
+ * Eq. 2 numerators X and denominator D, the Eq. 4 numerators
  * Y[w,s] = sum_t (F[t,S-1] - F'[t,S-1]) where F' replaces stage s by the
  * clipped baseline min(d, m) on every rank, the per-step leading stage with its
  * confidence (unique leader whose margin over the runner-up is

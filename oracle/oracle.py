@@ -1,7 +1,7 @@
 """CPU oracle for frontier accounting -- TEST INFRASTRUCTURE.
 
 Thin numpy wrapper over ``sforacle.c``, the literal restatement of the
-paper's definitions (Sec. 3 Eq. 1-2, Sec. 4 Eq. 3, App. A-C).  Only the test
+paper's definitions (Sec. 3 Eq. 1-2, Sec. 4 Eq. 4, App. A-C).  Only the test
 suite, ``__graft_entry__.smoke()`` and the benchmark's CPU-baseline leg may
 import this module; the product path never does.
 """

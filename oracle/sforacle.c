@@ -254,7 +254,7 @@ int sfo_label_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t
 
   /* step 1: windows' frontier numerators/denominator (Eq. 2) */
   if (rc == SFO_OK) rc = sfo_windows(d, T, R, S, 0, W, X, D, NULL, NULL, NULL);
-  /* step 2: per-rank window medians and the clipped-gain numerators (Eq. 3) */
+  /* step 2: per-rank window medians and the clipped-gain numerators (Eq. 4) */
   if (rc == SFO_OK) rc = sfo_window_median(d, T, R, S, W, m);
   if (rc == SFO_OK) rc = sfo_direct_gain(d, T, R, S, W, m, Y);
 
@@ -370,7 +370,7 @@ int sfo_label_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t
     if (amb_mask) amb_mask[w] = amb;
     for (int64_t s = 0; s < S; ++s) {
       if (share) share[w * S + s] = raw_only ? 0.0 : (double)Xw[s] / (double)Dw; /* A_s, Eq. 2 */
-      if (gain) gain[w * S + s] = raw_only ? 0.0 : (double)Yw[s] / (double)Dw;   /* G_s, Eq. 3 */
+      if (gain) gain[w * S + s] = raw_only ? 0.0 : (double)Yw[s] / (double)Dw;   /* G_s, Eq. 4 */
     }
     if (n_confident) n_confident[w] = e;
     if (n_switch) n_switch[w] = sw;

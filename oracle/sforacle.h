@@ -68,7 +68,7 @@ int sfo_topk(const int64_t* X, const int64_t* E, int64_t nW, int64_t S, int64_t 
    start at step 0 of d; the last may be short. m is [nW][R][S]. */
 int sfo_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W, int64_t* m);
 
-/* Sec. 4 Eq. 3 numerator, literally: for every step, replace stage s by
+/* Sec. 4 Eq. 4 numerator, literally: for every step, replace stage s by
    min(d, m) on every rank, recompute the frontier, accumulate F_S - F'_S. */
 int sfo_direct_gain(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W, const int64_t* m,
                     int64_t* Y);

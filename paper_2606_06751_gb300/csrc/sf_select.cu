@@ -1,6 +1,6 @@
 // sf_select.cu - the per-window kernels of libstagefrontier:
 //   * window_median: lower median of every (window, rank, stage) column
-//     (the per-rank window baseline of Sec. 4, Eq. 3);
+//     (the per-rank window baseline of Sec. 4, Eq. 4);
 //   * topk: top-k stages by X and (stage, rank) pairs by lead-rank credit E;
 //   * gates: App. C label gates, routing and ambiguity sets, fp64 shares/gains;
 //   * zero: clears accumulators the library owns the semantics of.

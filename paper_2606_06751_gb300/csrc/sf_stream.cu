@@ -4,7 +4,7 @@
 //     max-prefix frontier with its lowest attaining rank per boundary, the
 //     increments a[t,s], and the fused window aggregation (X, D, E, C, leading
 //     stage);
-//   * evidence pass (Sec. 4 Eq. 3): the same frontier plus, for every stage s,
+//   * evidence pass (Sec. 4 Eq. 4): the same frontier plus, for every stage s,
 //     the makespan after replacing s by the clipped per-rank window median,
 //     per-step leader confidence and the telemetry-quality sums (App. A).
 //

@@ -248,7 +248,7 @@ def test_topk_against_sorted(seed):
         assert list(t.pair_value[w]) == [-v for v, _, _ in pr] + [0] * (k - len(pr))
 
 
-# ---------------------------------------------------------------- median and gain (Eq. 3)
+# ---------------------------------------------------------------- median and gain (Eq. 4)
 
 @pytest.mark.parametrize("T,W", [(30, 10), (31, 10), (9, 4), (5, 16)])
 def test_median_is_lower_median(T, W):
