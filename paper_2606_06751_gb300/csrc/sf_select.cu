@@ -168,11 +168,6 @@ __global__ void __launch_bounds__(kMedThreads)
 // the column minimum stay in registers only when they fit 32 bits; wider
 // columns re-read shared memory on every radix pass.  Registers are capped so
 // three CTAs share an SM and one CTA's copy overlaps another's selection.
-__device__ __forceinline__ int64_t tile_at(const unsigned char* tile, int r, int c) {
-  const uint32_t off = uint32_t(r) * 64u + ((uint32_t(c >> 1) ^ ((uint32_t(r) >> 1) & 3u)) << 4) + (uint32_t(c & 1) << 3);
-  return *reinterpret_cast<const int64_t*>(tile + off);
-}
-
 template <int NPL>
 __global__ void __launch_bounds__(kMedThreads, 3)
     median_tma_kernel(const __grid_constant__ CUtensorMap map, int64_t T, int64_t RS, int64_t W,
@@ -211,37 +206,60 @@ __global__ void __launch_bounds__(kMedThreads, 3)
   }
   if (warp >= ncols) return;
   uint32_t* hist = hists + warp * kMedBins;
-  constexpr uint64_t kSign = 1ull << 63;
-  uint64_t lo = ~0ull, hi = 0;
+  // Row lane + 32 i of this warp's column: the 64-byte swizzle term depends
+  // only on (row >> 1) & 3 = (lane >> 1) & 3, so each lane has one base and a
+  // fixed 2048-byte stride.
+  const unsigned char* col = tile + lane * 64 + ((((warp >> 1) ^ ((lane >> 1) & 3)) << 4) | ((warp & 1) << 3));
+  // Order-preserving unsigned key of a signed value: flip the sign bit, i.e.
+  // bit 31 of the high word.  Most columns share one high word; then the
+  // whole selection runs on the 32-bit low words.
+  uint32_t xl[NPL];
+  uint32_t hmin = 0xffffffffu, hmax = 0, lmin = 0xffffffffu, lmax = 0;
 #pragma unroll
   for (int i = 0; i < NPL; ++i) {
-    const int row = lane + 32 * i;
-    if (row < n) {
-      const uint64_t u = static_cast<uint64_t>(tile_at(tile, row, warp)) ^ kSign;
-      lo = u < lo ? u : lo;
-      hi = u > hi ? u : hi;
+    if (lane + 32 * i < n) {
+      const uint2 v = *reinterpret_cast<const uint2*>(col + i * 2048);
+      const uint32_t h = v.y ^ 0x80000000u;
+      xl[i] = v.x;
+      hmin = min(hmin, h);
+      hmax = max(hmax, h);
+      lmin = min(lmin, v.x);
+      lmax = max(lmax, v.x);
+    } else {
+      xl[i] = 0;
     }
   }
-  lo = warp_min_u64(lo);
-  hi = warp_max_u64(hi);
+  hmin = __reduce_min_sync(kFull, hmin);
+  hmax = __reduce_max_sync(kFull, hmax);
   const uint32_t k = static_cast<uint32_t>((n - 1) / 2);
-  const uint64_t range = hi - lo;
-  const int nbits = range ? 64 - __clzll(static_cast<long long>(range)) : 0;
-  uint64_t ans;
-  if (nbits <= 32) {
-    uint32_t x[NPL];
+  uint64_t key;
+  if (hmin == hmax) {
+    lmin = __reduce_min_sync(kFull, lmin);
+    lmax = __reduce_max_sync(kFull, lmax);
+    const uint32_t range = lmax - lmin;
+    const int nbits = range ? 32 - __clz(static_cast<int>(range)) : 0;
 #pragma unroll
-    for (int i = 0; i < NPL; ++i) {
-      const int row = lane + 32 * i;
-      x[i] = row < n ? static_cast<uint32_t>((static_cast<uint64_t>(tile_at(tile, row, warp)) ^ kSign) - lo) : 0u;
-    }
-    ans = warp_radix_select<uint32_t, NPL>([&](int i) { return x[i]; }, n, nbits, k, hist, lane);
+    for (int i = 0; i < NPL; ++i) xl[i] -= lmin;  // padding slots are never read
+    const uint32_t ans = warp_radix_select<uint32_t, NPL>([&](int i) { return xl[i]; }, n, nbits, k, hist, lane);
+    key = (static_cast<uint64_t>(hmin) << 32) | (lmin + ans);
   } else {
-    ans = warp_radix_select<uint64_t, NPL>(
-        [&](int i) { return (static_cast<uint64_t>(tile_at(tile, lane + 32 * i, warp)) ^ kSign) - lo; }, n, nbits,
-        k, hist, lane);
+    constexpr uint64_t kSign = 1ull << 63;
+    auto ukey = [&](int i) { return static_cast<uint64_t>(*reinterpret_cast<const int64_t*>(col + i * 2048)) ^ kSign; };
+    uint64_t lo = ~0ull, hi = 0;
+#pragma unroll
+    for (int i = 0; i < NPL; ++i)
+      if (lane + 32 * i < n) {
+        const uint64_t u = ukey(i);
+        lo = u < lo ? u : lo;
+        hi = u > hi ? u : hi;
+      }
+    lo = warp_min_u64(lo);
+    hi = warp_max_u64(hi);
+    const uint64_t range = hi - lo;
+    const int nbits = range ? 64 - __clzll(static_cast<long long>(range)) : 0;
+    key = lo + warp_radix_select<uint64_t, NPL>([&](int i) { return ukey(i) - lo; }, n, nbits, k, hist, lane);
   }
-  if (lane == 0) m[w * RS + c0 + warp] = static_cast<int64_t>((lo + ans) ^ kSign);
+  if (lane == 0) m[w * RS + c0 + warp] = static_cast<int64_t>(key ^ (1ull << 63));
 }
 
 // Windows longer than 1024 steps: the same search, re-reading the column

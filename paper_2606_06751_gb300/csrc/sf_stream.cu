@@ -257,16 +257,47 @@ struct FrontierRows {
   }
 };
 
+constexpr int ceil_log2(int x) { return x <= 1 ? 0 : 1 + ceil_log2((x + 1) / 2); }
+
+// Evidence-pass maxima.  A row whose durations and medians are all below
+// 2^kNarrowBits (S * 2^kNarrowBits <= 2^31) is reduced in 32-bit arithmetic:
+// its prefixes stay below 2^31 and P_S - d + m below 2^32, so every value is
+// exact.  Other rows (long stages, invalid input) take the 64-bit path; the two
+// partial maxima are merged at the end of the step.
 template <int S>
 struct GainRows {
-  int64_t bf[S];  // max_r P[t,r,s]
-  int64_t bg[S];  // max_r (P[t,r,S-1] - max(0, d[t,r,s] - m[w,r,s]))
+  static constexpr int kNarrowBits = 31 - ceil_log2(S);
+  uint32_t nf[S], ng[S];  // narrow rows: max_r P[t,r,s], max_r (P_S - max(0, d - m))
+  int64_t bf[S], bg[S];   // wide rows
   __device__ __forceinline__ void init() {
 #pragma unroll
-    for (int s = 0; s < S; ++s) bf[s] = bg[s] = 0;
+    for (int s = 0; s < S; ++s) {
+      nf[s] = ng[s] = 0;
+      bf[s] = bg[s] = 0;
+    }
   }
   __device__ __forceinline__ int64_t row(const int64_t (&v)[S], const int64_t (&mr)[S], uint32_t& dor,
                                          uint32_t& tor) {
+    uint32_t big = 0;
+#pragma unroll
+    for (int s = 0; s < S; ++s)
+      big |= hi32(v[s]) | hi32(mr[s]) |
+             ((static_cast<uint32_t>(v[s]) | static_cast<uint32_t>(mr[s])) >> kNarrowBits);
+    if (big == 0) {
+      uint32_t P = 0;
+#pragma unroll
+      for (int s = 0; s < S; ++s) {
+        P += static_cast<uint32_t>(v[s]);
+        nf[s] = max(nf[s], P);
+      }
+#pragma unroll
+      for (int s = 0; s < S; ++s) {
+        // P_S - max(0, d - m) = min(P_S, P_S - d + m)
+        const uint32_t alt = min(P, P - static_cast<uint32_t>(v[s]) + static_cast<uint32_t>(mr[s]));
+        ng[s] = max(ng[s], alt);
+      }
+      return static_cast<int64_t>(P);
+    }
     int64_t P = 0;
 #pragma unroll
     for (int s = 0; s < S; ++s) {
@@ -283,6 +314,14 @@ struct GainRows {
       bg[s] = alt > bg[s] ? alt : bg[s];
     }
     return P;
+  }
+  __device__ __forceinline__ uint64_t F(int s) const {
+    const uint64_t w = static_cast<uint64_t>(bf[s]);
+    return w > nf[s] ? w : static_cast<uint64_t>(nf[s]);
+  }
+  __device__ __forceinline__ uint64_t G(int s) const {
+    const uint64_t w = static_cast<uint64_t>(bg[s]);
+    return w > ng[s] ? w : static_cast<uint64_t>(ng[s]);
   }
 };
 
@@ -468,8 +507,8 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
           int64_t myF = 0, myR = 0;
 #pragma unroll
           for (int s = 0; s < S; ++s) {
-            const uint64_t f = warp_max_u64(static_cast<uint64_t>(rs.bf[s]));
-            const uint64_t g = warp_max_u64(static_cast<uint64_t>(rs.bg[s]));
+            const uint64_t f = warp_max_u64(rs.F(s));
+            const uint64_t g = warp_max_u64(rs.G(s));
             if (lane == s) {
               myF = static_cast<int64_t>(f);
               myR = static_cast<int64_t>(g);
@@ -534,8 +573,8 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
           const uint64_t km = warp_max_u64(fr.key(s));
           if (lane == s) slot[s] = km;
         } else {
-          const uint64_t f = warp_max_u64(static_cast<uint64_t>(gr.bf[s]));
-          const uint64_t g = warp_max_u64(static_cast<uint64_t>(gr.bg[s]));
+          const uint64_t f = warp_max_u64(gr.F(s));
+          const uint64_t g = warp_max_u64(gr.G(s));
           if (lane == s) {
             slot[s] = f;
             slot[S + s] = g;
