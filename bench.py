@@ -1,9 +1,11 @@
 """Benchmark of the frontier-accounting hot path on GB300.
 
 One step = one pass of the whole path over one batch of synthetic telemetry:
-window aggregation fused into the frontier pass (Sec. 3 Eq. 1-2), top-k
-suspects, and the labeler (per-rank window medians, the clipped-gain evidence
-pass of Sec. 4 Eq. 4, App. C gates).  The default workload is the largest
+per-rank window medians, then one evidence pass that computes the frontier
+(Sec. 3 Eq. 1), the window aggregates with lead-rank credit (Eq. 2) and the
+clipped-gain numerators (Sec. 4 Eq. 4), then top-k suspects and the App. C
+gates.  The standalone frontier/aggregation pass (sf_window_aggregate) is timed
+beside the step as `frontier_pass`.  The default workload is the largest
 frontier-accounting configuration: 8192 ranks x 8 stages x 20000 steps of
 int64 ns (10.49 GB), 1000-step windows, top-5, labels.
 
@@ -215,18 +217,18 @@ class Pipeline:
         self.nW = sf.num_windows(0, T, W)
         nW = self.nW
         e = lambda shape, dt: torch.empty(shape, dtype=dt, device=dev)  # noqa: E731
-        self.win = sf.Windows(e((nW, S), torch.int64), e((nW,), torch.int64), e((nW, S, R), torch.int64),
-                              e((nW, S, R), torch.int32), e((T,), torch.uint8))
         self.top = sf.TopK(e((nW, k), torch.int32), e((nW, k), torch.int64), e((nW, k, 2), torch.int32),
                            e((nW, k), torch.int64))
         self.m = e((nW, R, S), torch.int64)
         self.ev = sf.Evidence(e((nW, S), torch.int64), e((nW, S), torch.int64), e((nW,), torch.int64),
-                              e((T,), torch.uint8), None)
+                              e((T,), torch.uint8), None, e((nW, S, R), torch.int64), e((nW, S, R), torch.int32))
         self.lab = sf.Labels(e((nW,), torch.int32), e((nW,), torch.int32), e((nW,), torch.int32),
                              e((nW, S), torch.float64), e((nW, S), torch.float64), e((nW,), torch.int32),
                              e((nW,), torch.int32))
+        self.win = sf.Windows(e((nW, S), torch.int64), e((nW,), torch.int64), e((nW, S, R), torch.int64),
+                              e((nW, S, R), torch.int32), e((T,), torch.uint8))
         self.status = sf.new_status(dev)
-        self.names = ["window_aggregate", "topk_suspects", "window_median", "direct_gain", "label_gates"]
+        self.names = ["window_median", "direct_gain", "topk_suspects", "label_gates"]
         self.events = None
 
     def step(self, d=None, timing=False):
@@ -234,39 +236,40 @@ class Pipeline:
         d = self.d if d is None else d
         ev = None
         if timing:
-            ev = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
             ev[0].record()
-        sf.sf_window_aggregate(d, w.W, X=self.win.X, D=self.win.D, E=self.win.E, C=self.win.C,
-                               step_lead=self.win.step_lead, status=self.status)
-        if timing:
-            ev[1].record()
-        sf.sf_topk_suspects(self.win.X, self.win.E, w.k, out=self.top)
-        if timing:
-            ev[2].record()
         sf.sf_window_median(d, w.W, m=self.m, status=self.status)
         if timing:
-            ev[3].record()
+            ev[1].record()
         sf.sf_direct_gain(d, w.W, self.m, out=self.ev, status=self.status)
         if timing:
-            ev[4].record()
+            ev[2].record()
+        sf.sf_topk_suspects(self.ev.X, self.ev.E, w.k, out=self.top)
+        if timing:
+            ev[3].record()
         sf.sf_label_gates(w.T, w.R, w.S, w.W, self.ev, out=self.lab)
         if timing:
-            ev[5].record()
+            ev[4].record()
             self.events.append(ev)
+
+    def aggregate(self):
+        """The standalone frontier pass with window aggregation (sf_window_aggregate)."""
+        self.sf.sf_window_aggregate(self.d, self.w.W, X=self.win.X, D=self.win.D, E=self.win.E, C=self.win.C,
+                                    step_lead=self.win.step_lead, status=self.status)
 
     def results(self):
         return [self.lab.labels, self.lab.route_mask, self.lab.amb_mask, self.lab.share, self.lab.gain,
-                self.top.stage, self.top.pair, self.top.pair_value, self.win.X, self.win.D]
+                self.top.stage, self.top.pair, self.top.pair_value, self.ev.X, self.ev.D]
 
     def algorithmic_bytes(self):
         w, nW = self.w, self.nW
         din = w.T * w.R * w.S * 8
         return {
-            "window_aggregate": din + nW * w.S * (w.R * 12 + 8) + nW * 8 + w.T,
-            "topk_suspects": nW * w.S * (w.R + 1) * 8 + nW * w.k * 24,
             "window_median": din + nW * w.R * w.S * 8,
-            "direct_gain": din + nW * w.R * w.S * 8 + nW * (2 * w.S + 1) * 8 + w.T,
+            "direct_gain": din + nW * w.R * w.S * 8 + nW * w.S * (w.R * 12 + 16) + nW * 8 + w.T,
+            "topk_suspects": nW * w.S * (w.R + 1) * 8 + nW * w.k * 24,
             "label_gates": nW * (2 * w.S + 1) * 8 + w.T + nW * (3 * 4 + 2 * w.S * 8),
+            "window_aggregate": din + nW * w.S * (w.R * 12 + 8) + nW * 8 + w.T,
         }
 
 
@@ -312,6 +315,9 @@ def run_ours(args):
     achieved = algo[dominant] / avg[dominant] / 1e9
     value = records * ws * args.steps / secs
 
+    # the standalone frontier/aggregation pass, timed on its own
+    agg_secs = timed_loop(pipe.aggregate, args.steps, args.warmup, ws, device, True) / args.steps
+
     # end to end: pinned host input copied in, results read back, every step
     outs = pipe.results()
     host_outs = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
@@ -330,6 +336,7 @@ def run_ours(args):
         return None
     kernels = {n: {"ms": round(avg[n] * 1e3, 4), "gbs": round(algo[n] / avg[n] / 1e9, 1),
                    "algorithmic_bytes": algo[n]} for n in pipe.names}
+    agg_gbs = algo["window_aggregate"] / agg_secs / 1e9
     traffic = profiled_traffic(dominant, w.name)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
@@ -345,6 +352,9 @@ def run_ours(args):
                      "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
                      "traffic": traffic},
         "kernels": kernels,
+        "frontier_pass": {"entry": "sf_window_aggregate", "ms": round(agg_secs * 1e3, 4),
+                          "gbs": round(agg_gbs, 1), "frac": round(agg_gbs / peak, 4),
+                          "records_per_s": records / agg_secs},
         "gpu_launches": int(launches * args.steps // (args.steps + args.warmup)),
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": w.nbytes, "d2h_bytes_per_step": d2h},
         "clocks": clk.summary(),

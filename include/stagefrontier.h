@@ -159,7 +159,9 @@ sf_status sf_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, in
 
 /*
  * sf_direct_gain - the evidence pass of the labeler (Sec. 4): per window the
- * Eq. 2 numerators X and denominator D, the Eq. 4 numerators
+ * Eq. 2 numerators X and denominator D, optionally the lead-rank credit E and
+ * lead counts C exactly as sf_window_aggregate defines them (so one pass over
+ * d serves both), the Eq. 4 numerators
  * Y[w,s] = sum_t (F[t,S-1] - F'[t,S-1]) where F' replaces stage s by the
  * clipped baseline min(d, m) on every rank, the per-step leading stage with its
  * confidence (unique leader whose margin over the runner-up is
@@ -168,6 +170,7 @@ sf_status sf_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, in
  *   wall       [T][R] step wall times (device, nullable).
  *   other_stage index of the residual stage, or -1.
  *   X [nW][S], Y [nW][S], D [nW] (device, required; overwritten).
+ *   E [nW][S][R] int64, C [nW][S][R] int32 (device, nullable; overwritten).
  *   step_lead  [T] leading stage | SF_STEP_CONFIDENT (device, required).
  *   quality    [nW][6] uint64 (device, nullable; overwritten): 128-bit sums
  *              (lo, hi) of the closure residual, the overlap error and the wall
@@ -177,8 +180,8 @@ sf_status sf_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, in
  */
 sf_status sf_direct_gain(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W,
                          const int64_t* m, const int64_t* wall, int32_t other_stage,
-                         sf_ratio eta_Q, int64_t* X, int64_t* Y, int64_t* D, uint8_t* step_lead,
-                         uint64_t* quality, uint32_t* status, cudaStream_t stream);
+                         sf_ratio eta_Q, int64_t* X, int64_t* Y, int64_t* D, int64_t* E, int32_t* C,
+                         uint8_t* step_lead, uint64_t* quality, uint32_t* status, cudaStream_t stream);
 
 /*
  * sf_label_gates - App. C gates per window from the evidence above: shares

@@ -192,18 +192,20 @@ sf_status sf_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, in
 
 sf_status sf_direct_gain(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W, const int64_t* m,
                          const int64_t* wall, int32_t other_stage, sf_ratio eta_Q, int64_t* X, int64_t* Y,
-                         int64_t* D, uint8_t* step_lead, uint64_t* quality, uint32_t* status,
-                         cudaStream_t stream) {
+                         int64_t* D, int64_t* E, int32_t* C, uint8_t* step_lead, uint64_t* quality,
+                         uint32_t* status, cudaStream_t stream) {
   if (!d || !m || !X || !Y || !D || !step_lead || !shape_ok(T, R, S) || W < 1 || W > 65536 ||
       other_stage < -1 || other_stage >= S || !ratio_ok(eta_Q))
     return SF_EINVAL;
   if (!aligned(d, 16) || !aligned(m, 8) || !aligned(wall, 8) || !aligned(X, 8) || !aligned(Y, 8) ||
-      !aligned(D, 8) || !aligned(quality, 8) || !aligned(status, 4))
+      !aligned(D, 8) || !aligned(E, 8) || !aligned(C, 4) || !aligned(quality, 8) || !aligned(status, 4))
     return SF_EINVAL_ALIGN;
   const int64_t nW = (T + W - 1) / W;
   cudaError_t e = launch_zero(X, size_t(nW) * S * 8, stream);
   if (e == cudaSuccess) e = launch_zero(Y, size_t(nW) * S * 8, stream);
   if (e == cudaSuccess) e = launch_zero(D, size_t(nW) * 8, stream);
+  if (e == cudaSuccess && E) e = launch_zero(E, size_t(nW) * S * R * 8, stream);
+  if (e == cudaSuccess && C) e = launch_zero(C, size_t(nW) * S * R * 4, stream);
   if (e == cudaSuccess && quality) e = launch_zero(quality, size_t(nW) * 6 * 8, stream);
   if (e != cudaSuccess) return SF_ECUDA;
   StreamJob j;
@@ -213,6 +215,8 @@ sf_status sf_direct_gain(const int64_t* d, int64_t T, int64_t R, int64_t S, int6
   j.S = S;
   j.X = X;
   j.D = D;
+  j.E = E;
+  j.C = C;
   j.step_lead = step_lead;
   j.W = W;
   j.gain = true;
@@ -289,7 +293,8 @@ sf_status sf_label_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, in
   uint8_t* sl = ws + L.sl;
   sf_status st = sf_window_median(d, T, R, S, W, m, status, stream);
   if (st != SF_OK) return st;
-  st = sf_direct_gain(d, T, R, S, W, m, wall, other_stage, cfg->eta_Q, Xw, Yw, Dw, sl, q, status, stream);
+  st = sf_direct_gain(d, T, R, S, W, m, wall, other_stage, cfg->eta_Q, Xw, Yw, Dw, nullptr, nullptr, sl, q,
+                      status, stream);
   if (st != SF_OK) return st;
   return sf_label_gates(T, R, S, W, Xw, Yw, Dw, sl, (wall || other_stage >= 0) ? q : nullptr, role, missing,
                         cfg, labels, route_mask, amb_mask, share, gain, nullptr, nullptr, stream);

@@ -35,6 +35,10 @@ __global__ void zero_kernel(uint32_t* __restrict__ p, size_t words) {
 constexpr int kMedCols = 8;
 constexpr int kMedThreads = kMedCols * 32;
 constexpr int kMedBins = 256;
+// Per-warp counters: 256 digit bins, then 32 per-lane discard slots that
+// non-matching and padding values increment instead of branching around the
+// atomic.  288 words = 1152 bytes keeps every warp's block 16-byte aligned.
+constexpr int kMedHistWords = kMedBins + 32;
 
 // k-th smallest (0-based) of the lane-strided values get(i) (row lane + 32 i,
 // valid while row < n), all below 2^nbits.  hist: this warp's 256 counters.
@@ -93,6 +97,79 @@ __device__ __forceinline__ U warp_radix_select(Get get, int n, int nbits, uint32
     rem -= below;
     prefix = (prefix << D) | static_cast<U>(digit);
     first = false;
+    __syncwarp();
+  }
+  return prefix;
+}
+
+// Shared-memory increment of one counter, issued only when `pred` is set
+// (explicitly predicated, so a warp never branches around it).
+__device__ __forceinline__ void red_shared_inc_if(uint32_t* counter, bool pred) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.u32 p, %1, 0;\n\t@p red.shared.add.u32 [%0], 1;\n\t}" ::"r"(smem_u32(counter)),
+      "r"(static_cast<uint32_t>(pred))
+      : "memory");
+}
+
+// Histogram scan of one radix pass: the digit d whose bin holds rank `rem`
+// among the counted values, and the count of values in lower bins.
+__device__ __forceinline__ void hist_find(const uint32_t* hist, uint32_t rem, int lane, uint32_t& digit,
+                                          uint32_t& below) {
+  const uint4 h0 = reinterpret_cast<const uint4*>(hist)[2 * lane];
+  const uint4 h1 = reinterpret_cast<const uint4*>(hist)[2 * lane + 1];
+  const uint32_t hb[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+  uint32_t sum = 0;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) sum += hb[j];
+  uint32_t incl = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t up = __shfl_up_sync(kFull, incl, o);
+    if (lane >= o) incl += up;
+  }
+  const uint32_t excl = incl - sum;
+  const int owner = __ffs(__ballot_sync(kFull, excl <= rem && rem < incl)) - 1;
+  uint32_t d = 0, bl = excl, c = excl;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const bool here = rem >= c && rem < c + hb[j];
+    d = here ? 8u * lane + j : d;
+    bl = here ? c : bl;
+    c += hb[j];
+  }
+  digit = __shfl_sync(kFull, d, owner);
+  below = __shfl_sync(kFull, bl, owner);
+}
+
+// The k-th smallest of the live values among x[i] (row lane + 32 i), by byte
+// digits, most significant first.  Padding slots must hold 0xffffffff: they
+// sort after every live value (all below 2^nbits, or tying only at the top
+// when nbits = 32), so counting them never moves the rank-k bin and no slot
+// needs a validity test.  The first pass counts every slot; later passes
+// count, with a predicated increment, only values whose higher bytes match the
+// digits chosen so far.
+template <int NPL>
+__device__ __forceinline__ uint32_t warp_select_bytes32(const uint32_t (&x)[NPL], int nbits, uint32_t k,
+                                                        uint32_t* hist, int lane) {
+  uint32_t prefix = 0, himask = 0, rem = k;
+  for (int b = (nbits + 7) / 8 - 1; b >= 0; --b) {
+    reinterpret_cast<uint4*>(hist)[2 * lane] = make_uint4(0, 0, 0, 0);
+    reinterpret_cast<uint4*>(hist)[2 * lane + 1] = make_uint4(0, 0, 0, 0);
+    __syncwarp();
+    const uint32_t sel = 0x4440u | uint32_t(b);  // __byte_perm selector: byte b of x, zero above
+    if (himask == 0) {
+#pragma unroll
+      for (int i = 0; i < NPL; ++i) atomicAdd(&hist[__byte_perm(x[i], 0, sel)], 1u);
+    } else {
+#pragma unroll
+      for (int i = 0; i < NPL; ++i) red_shared_inc_if(&hist[__byte_perm(x[i], 0, sel)], (x[i] & himask) == prefix);
+    }
+    __syncwarp();
+    uint32_t digit, below;
+    hist_find(hist, rem, lane, digit, below);
+    rem -= below;
+    prefix |= digit << (8 * b);
+    himask |= 0xffu << (8 * b);
     __syncwarp();
   }
   return prefix;
@@ -171,12 +248,13 @@ __global__ void __launch_bounds__(kMedThreads)
 template <int NPL>
 __global__ void __launch_bounds__(kMedThreads, 3)
     median_tma_kernel(const __grid_constant__ CUtensorMap map, int64_t T, int64_t RS, int64_t W,
-                      int64_t ngroups, int box_rows, int nbox, int64_t* __restrict__ m, uint32_t* status) {
+                      int64_t ngroups, int box_rows, int nbox, int tile_rows, int64_t* __restrict__ m,
+                      uint32_t* status) {
   extern __shared__ unsigned char smem_raw[];
   unsigned char* tile = align_1024(smem_raw);
-  const uint32_t tile_bytes = uint32_t(nbox) * uint32_t(box_rows) * 64u;
-  uint32_t* hists = reinterpret_cast<uint32_t*>(tile + tile_bytes);
-  uint64_t* bar = reinterpret_cast<uint64_t*>(hists + kMedCols * kMedBins);
+  const uint32_t tile_bytes = uint32_t(nbox) * uint32_t(box_rows) * 64u;  // bytes the copies write
+  uint32_t* hists = reinterpret_cast<uint32_t*>(tile + uint32_t(tile_rows) * 64u);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(hists + kMedCols * kMedHistWords);
   volatile int* abort = reinterpret_cast<volatile int*>(bar + 1);
   const int64_t w = blockIdx.x / ngroups;
   const int64_t c0 = (blockIdx.x % ngroups) * kMedCols;
@@ -205,7 +283,7 @@ __global__ void __launch_bounds__(kMedThreads, 3)
     return;
   }
   if (warp >= ncols) return;
-  uint32_t* hist = hists + warp * kMedBins;
+  uint32_t* hist = hists + warp * kMedHistWords;
   // Row lane + 32 i of this warp's column: the 64-byte swizzle term depends
   // only on (row >> 1) & 3 = (lane >> 1) & 3, so each lane has one base and a
   // fixed 2048-byte stride.
@@ -215,18 +293,17 @@ __global__ void __launch_bounds__(kMedThreads, 3)
   // whole selection runs on the 32-bit low words.
   uint32_t xl[NPL];
   uint32_t hmin = 0xffffffffu, hmax = 0, lmin = 0xffffffffu, lmax = 0;
+  const int live = n - lane;  // slot i holds a row of the window iff 32 i < live
 #pragma unroll
   for (int i = 0; i < NPL; ++i) {
-    if (lane + 32 * i < n) {
-      const uint2 v = *reinterpret_cast<const uint2*>(col + i * 2048);
+    const uint2 v = *reinterpret_cast<const uint2*>(col + i * 2048);  // in the tile even for padding slots
+    xl[i] = v.x;
+    if (32 * i < live) {
       const uint32_t h = v.y ^ 0x80000000u;
-      xl[i] = v.x;
       hmin = min(hmin, h);
       hmax = max(hmax, h);
       lmin = min(lmin, v.x);
       lmax = max(lmax, v.x);
-    } else {
-      xl[i] = 0;
     }
   }
   hmin = __reduce_min_sync(kFull, hmin);
@@ -239,8 +316,8 @@ __global__ void __launch_bounds__(kMedThreads, 3)
     const uint32_t range = lmax - lmin;
     const int nbits = range ? 32 - __clz(static_cast<int>(range)) : 0;
 #pragma unroll
-    for (int i = 0; i < NPL; ++i) xl[i] -= lmin;  // padding slots are never read
-    const uint32_t ans = warp_radix_select<uint32_t, NPL>([&](int i) { return xl[i]; }, n, nbits, k, hist, lane);
+    for (int i = 0; i < NPL; ++i) xl[i] = 32 * i < live ? xl[i] - lmin : 0xffffffffu;
+    const uint32_t ans = warp_select_bytes32<NPL>(xl, nbits, k, hist, lane);
     key = (static_cast<uint64_t>(hmin) << 32) | (lmin + ans);
   } else {
     constexpr uint64_t kSign = 1ull << 63;
@@ -527,12 +604,13 @@ template <int NPL>
 cudaError_t launch_median_tma(const CUtensorMap& map, int64_t T, int64_t RS, int64_t W, int64_t nW,
                               int64_t ngroups, int box_rows, int nbox, int64_t* m, uint32_t* status,
                               cudaStream_t stream) {
-  const size_t smem = 1024 + size_t(nbox) * box_rows * 64 + size_t(kMedCols) * kMedBins * 4 + 16;
+  const size_t tile_rows = std::max<size_t>(size_t(nbox) * box_rows, 32 * NPL);  // every slot's row is in the tile
+  const size_t smem = 1024 + tile_rows * 64 + size_t(kMedCols) * kMedHistWords * 4 + 16;
   cudaError_t e =
       cudaFuncSetAttribute(median_tma_kernel<NPL>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   median_tma_kernel<NPL><<<static_cast<unsigned>(nW * ngroups), kMedThreads, smem, stream>>>(
-      map, T, RS, W, ngroups, box_rows, nbox, m, status);
+      map, T, RS, W, ngroups, box_rows, nbox, static_cast<int>(tile_rows), m, status);
   return cudaGetLastError();
 }
 

@@ -145,11 +145,14 @@ __device__ __forceinline__ void finalize_frontier(const Params& p, int S, int64_
   }
 }
 
-// Evidence epilogue for step t.  Lane s < S holds F[t,s] and
+// Evidence epilogue for step t.  Lane s < S holds the packed frontier key
+// (F[t,s] << 16) | (65535 - lead[t,s]) and
 // Fr[t,s] = max_r (P[t,r,S-1] - max(0, d[t,r,s] - m[w,r,s])).
-__device__ __forceinline__ void finalize_gain(const Params& p, int S, int64_t t, int64_t F,
+__device__ __forceinline__ void finalize_gain(const Params& p, int S, int64_t t, uint64_t key,
                                               int64_t Fr, int lane, WinAcc& acc) {
   const bool valid = lane < S;
+  const int64_t F = valid ? static_cast<int64_t>(key >> 16) : 0;
+  const int32_t ld = valid ? 65535 - static_cast<int32_t>(key & 0xffffu) : 0;
   int64_t Fprev = __shfl_up_sync(kFull, F, 1);
   if (lane == 0) Fprev = 0;
   const int64_t a = valid ? F - Fprev : 0;
@@ -172,6 +175,12 @@ __device__ __forceinline__ void finalize_gain(const Params& p, int S, int64_t t,
   acc.x += a;
   acc.y += y;
   acc.dsum += FS;
+  if (valid && ld >= 0 && ld < p.R) {  // lead-rank credit (always in range for valid input)
+    const int64_t idx = (w * S + lane) * p.R + ld;
+    if (p.E && a != 0)
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.E[idx]), static_cast<unsigned long long>(a));
+    if (p.C) atomicAdd(&p.C[idx], 1);
+  }
 }
 
 // Telemetry-quality sums of one thread (App. A closure / overlap), flushed per window.
@@ -259,24 +268,32 @@ struct FrontierRows {
 
 constexpr int ceil_log2(int x) { return x <= 1 ? 0 : 1 + ceil_log2((x + 1) / 2); }
 
-// Evidence-pass maxima.  A row whose durations and medians are all below
-// 2^kNarrowBits (S * 2^kNarrowBits <= 2^31) is reduced in 32-bit arithmetic:
-// its prefixes stay below 2^31 and P_S - d + m below 2^32, so every value is
-// exact.  Other rows (long stages, invalid input) take the 64-bit path; the two
-// partial maxima are merged at the end of the step.
+// Evidence-pass maxima, with the frontier's lowest attaining rank.  A row
+// whose durations and medians are all below 2^kNarrowBits
+// (S * 2^kNarrowBits <= 2^31) is reduced in 32-bit arithmetic: its prefixes
+// stay below 2^31 and P_S - d + m below 2^32, so every value is exact.  Other
+// rows (long stages, invalid input) take the 64-bit path; the two partial
+// maxima are merged at the end of the step.  Rows arrive in increasing rank
+// order, so a strict '>' keeps the lowest rank on ties.
 template <int S>
 struct GainRows {
   static constexpr int kNarrowBits = 31 - ceil_log2(S);
-  uint32_t nf[S], ng[S];  // narrow rows: max_r P[t,r,s], max_r (P_S - max(0, d - m))
-  int64_t bf[S], bg[S];   // wide rows
+  uint32_t nf[S];        // narrow rows: 1 + max_r P[t,r,s] (0: none seen)
+  int32_t nr[S];         //   and the lowest rank attaining it
+  uint32_t ng[S];        //   max_r (P_S - max(0, d - m))
+  int64_t bf[S];         // wide rows: max_r P (-1: none seen)
+  int32_t br[S];
+  int64_t bg[S];
   __device__ __forceinline__ void init() {
 #pragma unroll
     for (int s = 0; s < S; ++s) {
       nf[s] = ng[s] = 0;
-      bf[s] = bg[s] = 0;
+      nr[s] = br[s] = 0;
+      bf[s] = -1;
+      bg[s] = 0;
     }
   }
-  __device__ __forceinline__ int64_t row(const int64_t (&v)[S], const int64_t (&mr)[S], uint32_t& dor,
+  __device__ __forceinline__ int64_t row(const int64_t (&v)[S], const int64_t (&mr)[S], int32_t r, uint32_t& dor,
                                          uint32_t& tor) {
     uint32_t big = 0;
 #pragma unroll
@@ -284,12 +301,16 @@ struct GainRows {
       big |= hi32(v[s]) | hi32(mr[s]) |
              ((static_cast<uint32_t>(v[s]) | static_cast<uint32_t>(mr[s])) >> kNarrowBits);
     if (big == 0) {
-      uint32_t P = 0;
+      uint32_t P1 = 1;  // prefix + 1
 #pragma unroll
       for (int s = 0; s < S; ++s) {
-        P += static_cast<uint32_t>(v[s]);
-        nf[s] = max(nf[s], P);
+        P1 += static_cast<uint32_t>(v[s]);
+        if (P1 > nf[s]) {
+          nf[s] = P1;
+          nr[s] = r;
+        }
       }
+      const uint32_t P = P1 - 1;
 #pragma unroll
       for (int s = 0; s < S; ++s) {
         // P_S - max(0, d - m) = min(P_S, P_S - d + m)
@@ -303,7 +324,10 @@ struct GainRows {
     for (int s = 0; s < S; ++s) {
       dor |= hi32(v[s]);
       P += v[s];
-      bf[s] = P > bf[s] ? P : bf[s];
+      if (P > bf[s]) {
+        bf[s] = P;
+        br[s] = r;
+      }
     }
     tor |= hi32(P);
 #pragma unroll
@@ -315,9 +339,13 @@ struct GainRows {
     }
     return P;
   }
-  __device__ __forceinline__ uint64_t F(int s) const {
-    const uint64_t w = static_cast<uint64_t>(bf[s]);
-    return w > nf[s] ? w : static_cast<uint64_t>(nf[s]);
+  // packed (F << 16) | (65535 - lead); 0 when this thread saw no row
+  __device__ __forceinline__ uint64_t key(int s) const {
+    const uint64_t kn =
+        nf[s] ? ((static_cast<uint64_t>(nf[s] - 1) << 16) | static_cast<uint64_t>(65535 - nr[s])) : 0ull;
+    const uint64_t kw =
+        bf[s] >= 0 ? ((static_cast<uint64_t>(bf[s]) << 16) | static_cast<uint64_t>(65535 - br[s])) : 0ull;
+    return kn > kw ? kn : kw;
   }
   __device__ __forceinline__ uint64_t G(int s) const {
     const uint64_t w = static_cast<uint64_t>(bg[s]);
@@ -499,22 +527,23 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
               int64_t v[S], mr[S];
               load_row<S, kSwz>(tile, q0 + r, v);
               load_global_row<S>(p.m + (w * p.R + r) * S, mr);
-              const int64_t total = rs.row(v, mr, dor, tor);
+              const int64_t total = rs.row(v, mr, r, dor, tor);
               if (p.quality)
                 qual_row(p, qa, t, r, total, p.other_stage >= 0 ? pick<S>(v, p.other_stage) : 0, dor);
             }
           }
-          int64_t myF = 0, myR = 0;
+          uint64_t myK = 0;
+          int64_t myR = 0;
 #pragma unroll
           for (int s = 0; s < S; ++s) {
-            const uint64_t f = warp_max_u64(rs.F(s));
+            const uint64_t f = warp_max_u64(rs.key(s));
             const uint64_t g = warp_max_u64(rs.G(s));
             if (lane == s) {
-              myF = static_cast<int64_t>(f);
+              myK = f;
               myR = static_cast<int64_t>(g);
             }
           }
-          finalize_gain(p, S, t, myF, myR, lane, acc);
+          finalize_gain(p, S, t, myK, myR, lane, acc);
         }
       }
       __syncwarp();
@@ -556,7 +585,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
               int64_t v[S], mr[S];
               load_row<S, kSwz>(tile, r - rank_tile0, v);
               load_row<S, kSwz>(tile + kR1StageBytes / 2, r - rank_tile0, mr);  // m tile of the same ranks
-              const int64_t total = gr.row(v, mr, dor, tor);
+              const int64_t total = gr.row(v, mr, r, dor, tor);
               if (p.quality)
                 qual_row(p, qa, t, r, total, p.other_stage >= 0 ? pick<S>(v, p.other_stage) : 0, dor);
             }
@@ -573,7 +602,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
           const uint64_t km = warp_max_u64(fr.key(s));
           if (lane == s) slot[s] = km;
         } else {
-          const uint64_t f = warp_max_u64(gr.F(s));
+          const uint64_t f = warp_max_u64(gr.key(s));
           const uint64_t g = warp_max_u64(gr.G(s));
           if (lane == s) {
             slot[s] = f;
@@ -593,7 +622,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
           }
         }
         if constexpr (!GAIN) finalize_frontier(p, S, t, v0, lane, acc);
-        else finalize_gain(p, S, t, static_cast<int64_t>(v0), static_cast<int64_t>(v1), lane, acc);
+        else finalize_gain(p, S, t, v0, static_cast<int64_t>(v1), lane, acc);
       }
       buf ^= 1;
     }
@@ -629,7 +658,7 @@ __global__ void __launch_bounds__(kGenThreads)
     int64_t b0[32], b1[32];
     int32_t br[32];
     for (int s = 0; s < S; ++s) {
-      b0[s] = GAIN ? 0 : -1;
+      b0[s] = -1;
       b1[s] = 0;
       br[s] = 0;
     }
@@ -658,9 +687,8 @@ __global__ void __launch_bounds__(kGenThreads)
       }
     }
     for (int s = 0; s < S; ++s) {
-      uint64_t k0;
-      if (GAIN) k0 = static_cast<uint64_t>(b0[s]);
-      else k0 = b0[s] < 0 ? 0ull : (static_cast<uint64_t>(b0[s]) << 16) | static_cast<uint64_t>(65535 - br[s]);
+      const uint64_t k0 =
+          b0[s] < 0 ? 0ull : (static_cast<uint64_t>(b0[s]) << 16) | static_cast<uint64_t>(65535 - br[s]);
       const uint64_t m0 = warp_max_u64(k0);
       const uint64_t m1 = GAIN ? warp_max_u64(static_cast<uint64_t>(b1[s])) : 0;
       if (lane == 0) {
@@ -676,7 +704,7 @@ __global__ void __launch_bounds__(kGenThreads)
           v0 = red[ww][lane] > v0 ? red[ww][lane] : v0;
           v1 = red[ww][32 + lane] > v1 ? red[ww][32 + lane] : v1;
         }
-      if (GAIN) finalize_gain(p, S, t, static_cast<int64_t>(v0), static_cast<int64_t>(v1), lane, acc);
+      if (GAIN) finalize_gain(p, S, t, v0, static_cast<int64_t>(v1), lane, acc);
       else finalize_frontier(p, S, t, v0, lane, acc);
     }
     __syncthreads();

@@ -54,7 +54,7 @@ def _load():
         "sf_window_aggregate": [P, I, I, I, I, I, P, P, P, P, P, I32, P, S],
         "sf_topk_suspects": [P, P, I, I, I, I32, P, P, P, P, S],
         "sf_window_median": [P, I, I, I, I, P, P, S],
-        "sf_direct_gain": [P, I, I, I, I, P, P, I32, Ratio, P, P, P, P, P, P, S],
+        "sf_direct_gain": [P, I, I, I, I, P, P, I32, Ratio, P, P, P, P, P, P, P, P, S],
         "sf_label_gates": [I, I, I, I, P, P, P, P, P, P, P, ctypes.POINTER(LabelConfig), P, P, P, P,
                            P, P, P, S],
         "sf_label_windows": [P, I, I, I, I, P, P, P, I32, ctypes.POINTER(LabelConfig), P,
@@ -218,19 +218,24 @@ class Evidence:
     D: torch.Tensor
     step_lead: torch.Tensor
     quality: Optional[torch.Tensor]
+    E: Optional[torch.Tensor] = None
+    C: Optional[torch.Tensor] = None
 
 
 def sf_direct_gain(d, W: int, m, wall=None, other_stage: int = -1, eta_Q=(1, 20), out: Optional[Evidence] = None,
-                   status=None, stream=None):
+                   lead_credit: bool = False, status=None, stream=None):
     T, R, S = _d3(d)
     nW = (T + W - 1) // W
     if out is None:
         q = _empty((nW, 6), torch.uint64, d) if (wall is not None or other_stage >= 0) else None
         out = Evidence(_empty((nW, S), torch.int64, d), _empty((nW, S), torch.int64, d),
                        _empty((nW,), torch.int64, d), _empty((T,), torch.uint8, d), q)
+        if lead_credit:
+            out.E = _empty((nW, S, R), torch.int64, d)
+            out.C = _empty((nW, S, R), torch.int32, d)
     _check(_lib.sf_direct_gain(_p(d), T, R, S, W, _p(m), _p(wall), other_stage, Ratio(*eta_Q), _p(out.X),
-                               _p(out.Y), _p(out.D), _p(out.step_lead), _p(out.quality), _p(status),
-                               _stream(stream)), "sf_direct_gain")
+                               _p(out.Y), _p(out.D), _p(out.E), _p(out.C), _p(out.step_lead), _p(out.quality),
+                               _p(status), _stream(stream)), "sf_direct_gain")
     return out
 
 

@@ -90,10 +90,12 @@ def test_host_validation(sf):
               FAKE, FAKE, None, None, None, None, None, None, None) == sf.SF_EINVAL_ALIGN
     # evidence pass: bad eta ratio and residual stage index
     dg = L.sf_direct_gain
-    assert dg(FAKE, 10, 4, 4, 5, FAKE, None, -1, sf.Ratio(1, 0), FAKE, FAKE, FAKE, FAKE, None, None,
-              None) == sf.SF_EINVAL
-    assert dg(FAKE, 10, 4, 4, 5, FAKE, None, -2, sf.Ratio(1, 20), FAKE, FAKE, FAKE, FAKE, None, None,
-              None) == sf.SF_EINVAL
+    assert dg(FAKE, 10, 4, 4, 5, FAKE, None, -1, sf.Ratio(1, 0), FAKE, FAKE, FAKE, None, None, FAKE, None,
+              None, None) == sf.SF_EINVAL
+    assert dg(FAKE, 10, 4, 4, 5, FAKE, None, -2, sf.Ratio(1, 20), FAKE, FAKE, FAKE, None, None, FAKE, None,
+              None, None) == sf.SF_EINVAL
+    assert dg(FAKE, 10, 4, 4, 5, FAKE, None, -1, sf.Ratio(1, 20), FAKE, FAKE, FAKE, FAKE + 4, None, FAKE,
+              None, None, None) == sf.SF_EINVAL_ALIGN
     assert L.sf_window_median(FAKE, 10, 4, 4, 0, FAKE, None, None) == sf.SF_EINVAL
     # nothing was launched by any of the rejected calls
     assert sf.launch_count() == 0

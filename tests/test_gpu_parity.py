@@ -89,7 +89,7 @@ def test_long_ranges_reuse_ring(sf, T, R, S):
     f = sf.sf_frontier(d, status=st)
     g = sf.sf_window_aggregate(d, W, status=st)
     m = sf.sf_window_median(d, W)
-    ev = sf.sf_direct_gain(d, W, m, status=st)
+    ev = sf.sf_direct_gain(d, W, m, lead_credit=True, status=st)
     torch.cuda.synchronize()
     assert int(st.item()) == 0
     assert np.array_equal(host(f.a), o.a) and np.array_equal(host(f.lead), o.lead)
@@ -97,6 +97,7 @@ def test_long_ranges_reuse_ring(sf, T, R, S):
     for name in ("X", "D", "E", "C", "step_lead"):
         assert np.array_equal(host(getattr(g, name)), getattr(ow, name)), name
     assert np.array_equal(host(ev.X), ow.X) and np.array_equal(host(ev.D), ow.D)
+    assert np.array_equal(host(ev.E), ow.E) and np.array_equal(host(ev.C), ow.C)
     assert np.array_equal(host(ev.step_lead) & 31, ow.step_lead)
     # gain numerators on the first two windows (the literal oracle is S x slower)
     m2 = O.window_median(d_np[:2 * W], W)
@@ -170,10 +171,11 @@ def test_direct_gain_parity(sf, T, R, S, W):
     m_np = O.window_median(d_np, W)
     Y = O.direct_gain(d_np, W, m_np)
     ow = O.windows(d_np, W)
-    ev = sf.sf_direct_gain(dev(d_np), W, dev(m_np))
+    ev = sf.sf_direct_gain(dev(d_np), W, dev(m_np), lead_credit=True)
     assert np.array_equal(host(ev.Y), Y)
     assert np.array_equal(host(ev.D), [ow.D[w] for w in range(len(ow.D))])
     assert np.array_equal(host(ev.X), ow.X)
+    assert np.array_equal(host(ev.E), ow.E) and np.array_equal(host(ev.C), ow.C)
     assert np.array_equal(host(ev.step_lead) & 31, ow.step_lead)
 
 
