@@ -6,6 +6,8 @@
 //   * zero: clears accumulators the library owns the semantics of.
 #include <algorithm>
 
+#include <cooperative_groups.h>
+
 #include "sf_device.cuh"
 #include "sf_launch.h"
 
@@ -405,21 +407,31 @@ __device__ VI block_best(VI x, VI* sm) {
   return r;
 }
 
-__global__ void __launch_bounds__(kTopThreads)
-    topk_kernel(const int64_t* __restrict__ X, const int64_t* __restrict__ E, int64_t S, int64_t R,
-                int k, int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair,
-                int64_t* top_pair_value) {
+// A window's (stage, rank) entries are split over a cluster of kTopCluster
+// CTAs.  Each CTA finds the top k of its slice (k rounds of a block arg-max,
+// each round taking the best entry ranked after the previous pick), parks them
+// in its shared memory, and the cluster's first CTA merges the cluster's
+// k x kTopCluster candidates read through distributed shared memory.
+constexpr int kTopCluster = 8;
+
+__global__ void __cluster_dims__(kTopCluster, 1, 1) __launch_bounds__(kTopThreads)
+    topk_kernel(const int64_t* __restrict__ X, const int64_t* __restrict__ E, int64_t S, int64_t R, int k,
+                int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair, int64_t* top_pair_value) {
+  namespace cg = cooperative_groups;
+  cg::cluster_group cluster = cg::this_cluster();
   __shared__ VI sm[kTopThreads / 32];
-  const int64_t w = blockIdx.x;
-  if (threadIdx.x < 32 && (top_stage || top_stage_value)) {
+  __shared__ VI cand[32];
+  const unsigned part = cluster.block_rank();
+  const int64_t w = blockIdx.x / kTopCluster;
+  if (part == 0 && threadIdx.x < 32 && (top_stage || top_stage_value)) {
     const int lane = threadIdx.x;
     const int64_t v = lane < S ? X[w * S + lane] : 0;
     bool taken = false;
     for (int i = 0; i < k; ++i) {
-      const uint64_t cand = (!taken && lane < S && v > 0) ? static_cast<uint64_t>(v) : 0ull;
-      const uint64_t mx = warp_max_u64(cand);
+      const uint64_t c = (!taken && lane < S && v > 0) ? static_cast<uint64_t>(v) : 0ull;
+      const uint64_t mx = warp_max_u64(c);
       int who = -1;
-      if (mx != 0) who = __ffs(__ballot_sync(kFull, cand == mx)) - 1;  // lowest stage among equals
+      if (mx != 0) who = __ffs(__ballot_sync(kFull, c == mx)) - 1;  // lowest stage among equals
       if (lane == who) taken = true;
       if (lane == 0) {
         if (top_stage) top_stage[w * k + i] = who;
@@ -427,35 +439,44 @@ __global__ void __launch_bounds__(kTopThreads)
       }
     }
   }
-  if (E == nullptr || (top_pair == nullptr && top_pair_value == nullptr)) return;
+  if (E == nullptr || (top_pair == nullptr && top_pair_value == nullptr)) return;  // uniform over the cluster
   const int64_t n = S * R;
+  const int64_t chunk = (n + kTopCluster - 1) / kTopCluster;
+  const int64_t lo = part * chunk, hi = lo + chunk < n ? lo + chunk : n;
   const int64_t* Ew = E + w * n;
   VI prev{INT64_MAX, -1};
   for (int i = 0; i < k; ++i) {
     VI best{0, INT64_MAX};
-    for (int64_t j = threadIdx.x; j < n; j += kTopThreads) {
-      const VI c{Ew[j], j};
-      if (c.v <= 0 || !before(prev, c)) continue;  // only entries ranked after the last pick
-      if (before(c, best)) best = c;
-    }
+    if (prev.v > 0)
+      for (int64_t j = lo + threadIdx.x; j < hi; j += kTopThreads) {
+        const VI c{Ew[j], j};
+        if (c.v > 0 && before(prev, c) && before(c, best)) best = c;  // ranked after the last pick
+      }
     best = block_best(best, sm);
-    if (threadIdx.x == 0) {
-      const bool ok = best.v > 0;
-      if (top_pair) {
-        top_pair[(w * k + i) * 2 + 0] = ok ? static_cast<int32_t>(best.i / R) : -1;
-        top_pair[(w * k + i) * 2 + 1] = ok ? static_cast<int32_t>(best.i % R) : -1;
-      }
-      if (top_pair_value) top_pair_value[w * k + i] = ok ? best.v : 0;
-    }
-    if (best.v <= 0) {
-      for (int ii = i + 1 + threadIdx.x; ii < k; ii += kTopThreads) {
-        if (top_pair) top_pair[(w * k + ii) * 2 + 0] = top_pair[(w * k + ii) * 2 + 1] = -1;
-        if (top_pair_value) top_pair_value[w * k + ii] = 0;
-      }
-      break;
-    }
-    prev = best;
+    if (threadIdx.x == 0) cand[i] = best;
+    prev = best.v > 0 ? best : VI{0, INT64_MAX};
   }
+  cluster.sync();
+  if (part == 0) {
+    const int t = threadIdx.x;
+    VI mine{0, INT64_MAX};
+    if (t < kTopCluster * k) mine = cluster.map_shared_rank(cand, static_cast<unsigned>(t / k))[t % k];
+    prev = VI{INT64_MAX, -1};
+    for (int i = 0; i < k; ++i) {
+      VI c = (mine.v > 0 && before(prev, mine)) ? mine : VI{0, INT64_MAX};
+      c = block_best(c, sm);
+      if (threadIdx.x == 0) {
+        const bool ok = c.v > 0;
+        if (top_pair) {
+          top_pair[(w * k + i) * 2 + 0] = ok ? static_cast<int32_t>(c.i / R) : -1;
+          top_pair[(w * k + i) * 2 + 1] = ok ? static_cast<int32_t>(c.i % R) : -1;
+        }
+        if (top_pair_value) top_pair_value[w * k + i] = ok ? c.v : 0;
+      }
+      prev = c.v > 0 ? c : VI{0, INT64_MAX};
+    }
+  }
+  cluster.sync();  // the other CTAs' candidates stay in place until the merge has read them
 }
 
 // ---------------------------------------------------------------------------
@@ -668,8 +689,8 @@ cudaError_t launch_topk(const int64_t* X, const int64_t* E, int64_t nW, int64_t 
                         int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair,
                         int64_t* top_pair_value, cudaStream_t stream) {
   count_launch();
-  topk_kernel<<<static_cast<unsigned>(nW), kTopThreads, 0, stream>>>(X, E, S, R, k, top_stage, top_stage_value,
-                                                                     top_pair, top_pair_value);
+  topk_kernel<<<static_cast<unsigned>(nW * kTopCluster), kTopThreads, 0, stream>>>(
+      X, E, S, R, k, top_stage, top_stage_value, top_pair, top_pair_value);
   return cudaGetLastError();
 }
 

@@ -278,6 +278,8 @@ constexpr int ceil_log2(int x) { return x <= 1 ? 0 : 1 + ceil_log2((x + 1) / 2);
 template <int S>
 struct GainRows {
   static constexpr int kNarrowBits = 31 - ceil_log2(S);
+  // With S > 10 the doubled state would spill; those shapes use the 64-bit path only.
+  static constexpr bool kNarrow = S <= 10;
   uint32_t nf[S];        // narrow rows: 1 + max_r P[t,r,s] (0: none seen)
   int32_t nr[S];         //   and the lowest rank attaining it
   uint32_t ng[S];        //   max_r (P_S - max(0, d - m))
@@ -295,11 +297,13 @@ struct GainRows {
   }
   __device__ __forceinline__ int64_t row(const int64_t (&v)[S], const int64_t (&mr)[S], int32_t r, uint32_t& dor,
                                          uint32_t& tor) {
-    uint32_t big = 0;
+    uint32_t big = kNarrow ? 0u : 1u;
+    if (kNarrow) {
 #pragma unroll
-    for (int s = 0; s < S; ++s)
-      big |= hi32(v[s]) | hi32(mr[s]) |
-             ((static_cast<uint32_t>(v[s]) | static_cast<uint32_t>(mr[s])) >> kNarrowBits);
+      for (int s = 0; s < S; ++s)
+        big |= hi32(v[s]) | hi32(mr[s]) |
+               ((static_cast<uint32_t>(v[s]) | static_cast<uint32_t>(mr[s])) >> kNarrowBits);
+    }
     if (big == 0) {
       uint32_t P1 = 1;  // prefix + 1
 #pragma unroll
