@@ -222,6 +222,40 @@ sf_status sf_label_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, in
                            int64_t* Y, int64_t* D, uint32_t* status, cudaStream_t stream);
 
 /*
+ * sf_stream_windows - the whole hot path over a tensor that lives in HOST
+ * memory: the steps are cut into chunks of chunk_steps steps (a multiple of
+ * W, so every chunk holds whole windows); each chunk is copied host->device on
+ * `copy_stream` into one of two device staging buffers and then, on
+ * `stream`, gets sf_window_median, sf_direct_gain (with lead-rank credit when
+ * E/C are given), sf_topk_suspects and sf_label_gates, its windows written to
+ * the output rows they belong to.  The copy of the next chunk overlaps the
+ * computation of the current one when h_d is page-locked and the two streams
+ * differ.  This is the SURVEY's chunked streaming of the largest workload
+ * (Sec. 5's window-boundary delivery of rank vectors, here host to GPU).
+ *   h_d        [T][R][S] host, 16-byte aligned (page-locked for overlap).
+ *   staging    device, >= sf_stream_windows_staging_size(T, R, S, chunk_steps)
+ *              bytes, 16-byte aligned: two chunk buffers.
+ *   workspace  device, >= sf_label_windows_workspace_size(min(chunk_steps, T),
+ *              R, S, W) bytes: one chunk's medians and step leaders.
+ *   outputs (device) indexed by global window: X, Y [nW][S], D [nW] required;
+ *   E [nW][S][R], C [nW][S][R], top_stage, top_pair [nW][k][2],
+ *   top_pair_value [nW][k], share, gain [nW][S] nullable; labels, route_mask,
+ *   amb_mask [nW] required.  No telemetry-quality or role inputs.
+ * The call creates and releases four CUDA events; it allocates no memory.
+ * Returns when everything is enqueued.
+ */
+sf_status sf_stream_windows(const int64_t* h_d, int64_t T, int64_t R, int64_t S, int64_t W, int32_t k,
+                            int64_t chunk_steps, const sf_label_config* cfg, int64_t* staging,
+                            size_t staging_bytes, void* workspace, size_t workspace_bytes, int64_t* X,
+                            int64_t* Y, int64_t* D, int64_t* E, int32_t* C, int32_t* top_stage,
+                            int32_t* top_pair, int64_t* top_pair_value, uint32_t* labels,
+                            uint32_t* route_mask, uint32_t* amb_mask, double* share, double* gain,
+                            uint32_t* status, cudaStream_t stream, cudaStream_t copy_stream);
+
+/* Device staging bytes sf_stream_windows needs; 0 on bad arguments. */
+size_t sf_stream_windows_staging_size(int64_t T, int64_t R, int64_t S, int64_t chunk_steps);
+
+/*
  * sf_label_windows_noalloc - sf_label_windows for callers that cannot
  * allocate device memory.  The paper has no counterpart; this is a
  * deployment variant of the labeler above.  It exists because an always-on

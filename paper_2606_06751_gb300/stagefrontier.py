@@ -61,6 +61,8 @@ def _load():
                              ctypes.c_size_t, P, P, P, P, P, P, P, P, P, S],
         "sf_label_windows_noalloc": [P, I, I, I, I, P, P, P, I32, ctypes.POINTER(LabelConfig), P, P, P,
                                      P, P, P, P, P, P, S],
+        "sf_stream_windows": [P, I, I, I, I, I32, I, ctypes.POINTER(LabelConfig), P, ctypes.c_size_t, P,
+                              ctypes.c_size_t, P, P, P, P, P, P, P, P, P, P, P, P, P, P, S, S],
     }
     for name, argt in sigs.items():
         f = getattr(L, name)
@@ -76,6 +78,8 @@ def _load():
     L.sf_label_config_default.restype = None
     L.sf_label_windows_workspace_size.argtypes = [I, I, I, I]
     L.sf_label_windows_workspace_size.restype = ctypes.c_size_t
+    L.sf_stream_windows_staging_size.argtypes = [I, I, I, I]
+    L.sf_stream_windows_staging_size.restype = ctypes.c_size_t
     return L
 
 
@@ -318,3 +322,58 @@ def sf_label_windows_noalloc(d, W: int, role=None, missing=None, wall=None, othe
                                          _p(out.Y), _p(out.D), _p(status), _stream(stream)),
            "sf_label_windows_noalloc")
     return out
+
+
+@dataclass
+class Streamed:
+    X: torch.Tensor
+    Y: torch.Tensor
+    D: torch.Tensor
+    E: Optional[torch.Tensor]
+    C: Optional[torch.Tensor]
+    top_stage: torch.Tensor
+    top_pair: Optional[torch.Tensor]
+    top_pair_value: Optional[torch.Tensor]
+    labels: torch.Tensor
+    route_mask: torch.Tensor
+    amb_mask: torch.Tensor
+    share: torch.Tensor
+    gain: torch.Tensor
+
+
+class StreamBuffers:
+    """Device staging, workspace and outputs for sf_stream_windows, reusable across calls."""
+
+    def __init__(self, T: int, R: int, S: int, W: int, k: int, chunk_steps: int, device, lead_credit=True):
+        nW = (T + W - 1) // W
+        e = lambda shape, dt: torch.empty(shape, dtype=dt, device=device)  # noqa: E731
+        self.shape = (T, R, S, W, k, chunk_steps)
+        self.staging = e((int(_lib.sf_stream_windows_staging_size(T, R, S, chunk_steps)),), torch.uint8)
+        self.workspace = e((workspace_size(min(chunk_steps, T), R, S, W),), torch.uint8)
+        self.out = Streamed(e((nW, S), torch.int64), e((nW, S), torch.int64), e((nW,), torch.int64),
+                            e((nW, S, R), torch.int64) if lead_credit else None,
+                            e((nW, S, R), torch.int32) if lead_credit else None,
+                            e((nW, k), torch.int32), e((nW, k, 2), torch.int32) if lead_credit else None,
+                            e((nW, k), torch.int64) if lead_credit else None,
+                            e((nW,), torch.int32), e((nW,), torch.int32), e((nW,), torch.int32),
+                            e((nW, S), torch.float64), e((nW, S), torch.float64))
+
+
+def sf_stream_windows(h_d: torch.Tensor, W: int, k: int, chunk_steps: int, bufs: StreamBuffers = None,
+                      cfg=None, status=None, stream=None, copy_stream=None) -> Streamed:
+    """h_d: [T][R][S] int64 CPU tensor (pin it for copy/compute overlap)."""
+    if h_d.is_cuda or h_d.dtype != torch.int64 or not h_d.is_contiguous() or h_d.dim() != 3:
+        raise TypeError("h_d must be a contiguous [T][R][S] int64 host tensor")
+    T, R, S = h_d.shape
+    cfg = cfg if cfg is not None else default_config()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    if bufs is None:
+        bufs = StreamBuffers(T, R, S, W, k, chunk_steps, dev)
+    o = bufs.out
+    cs = copy_stream if copy_stream is not None else (stream if stream is not None else torch.cuda.current_stream())
+    _check(_lib.sf_stream_windows(h_d.data_ptr(), T, R, S, W, k, chunk_steps, ctypes.byref(cfg),
+                                  _p(bufs.staging), bufs.staging.numel(), _p(bufs.workspace), bufs.workspace.numel(),
+                                  _p(o.X), _p(o.Y), _p(o.D), _p(o.E), _p(o.C), _p(o.top_stage), _p(o.top_pair),
+                                  _p(o.top_pair_value), _p(o.labels), _p(o.route_mask), _p(o.amb_mask), _p(o.share),
+                                  _p(o.gain), _p(status), _stream(stream), cs.cuda_stream), "sf_stream_windows")
+    return o
