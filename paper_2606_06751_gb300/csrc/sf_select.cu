@@ -294,22 +294,33 @@ __global__ void __launch_bounds__(kMedThreads, 3)
   // bit 31 of the high word.  Most columns share one high word; then the
   // whole selection runs on the 32-bit low words.
   uint32_t xl[NPL];
-  uint32_t hmin = 0xffffffffu, hmax = 0, lmin = 0xffffffffu, lmax = 0;
   const int live = n - lane;  // slot i holds a row of the window iff 32 i < live
+  // Low-word min/max over pairs of slots with 3-input min/max; a padding slot
+  // repeats row 0's value (row 0 is always in the window) so it cannot move
+  // either.  High words only need to agree: OR-accumulate their differences
+  // from row 0's high word.
+  const uint2 own0 = *reinterpret_cast<const uint2*>(col);  // lane 0's first slot is row 0
+  const uint32_t ref_x = __shfl_sync(kFull, own0.x, 0);
+  const uint32_t ref_y = __shfl_sync(kFull, own0.y, 0);
+  uint32_t lmin = ref_x, lmax = ref_x, hdiff = 0;
 #pragma unroll
   for (int i = 0; i < NPL; ++i) {
     const uint2 v = *reinterpret_cast<const uint2*>(col + i * 2048);  // in the tile even for padding slots
-    xl[i] = v.x;
-    if (32 * i < live) {
-      const uint32_t h = v.y ^ 0x80000000u;
-      hmin = min(hmin, h);
-      hmax = max(hmax, h);
-      lmin = min(lmin, v.x);
-      lmax = max(lmax, v.x);
-    }
+    const bool ok = 32 * i < live;
+    xl[i] = ok ? v.x : ref_x;
+    hdiff |= ok ? (v.y ^ ref_y) : 0u;
   }
-  hmin = __reduce_min_sync(kFull, hmin);
-  hmax = __reduce_max_sync(kFull, hmax);
+#pragma unroll
+  for (int i = 0; i + 1 < NPL; i += 2) {
+    lmin = __vimin3_u32(lmin, xl[i], xl[i + 1]);
+    lmax = __vimax3_u32(lmax, xl[i], xl[i + 1]);
+  }
+  if (NPL & 1) {
+    lmin = min(lmin, xl[NPL - 1]);
+    lmax = max(lmax, xl[NPL - 1]);
+  }
+  const bool narrow = __all_sync(kFull, hdiff == 0);
+  const uint32_t hmin = ref_y ^ 0x80000000u, hmax = narrow ? hmin : hmin + 1u;
   const uint32_t k = static_cast<uint32_t>((n - 1) / 2);
   uint64_t key;
   if (hmin == hmax) {
