@@ -82,6 +82,12 @@ int64_t sf_num_windows(int64_t t0, int64_t T, int64_t W);
 /* Kernels this library has launched since it was loaded (all entry points). */
 uint64_t sf_launch_count(void);
 
+/* Self-test of the device-side bounded waits every pipelined kernel uses: a
+   one-CTA kernel waits on a barrier phase that never completes, gives up after
+   limit_ns (0 < limit_ns <= 2 s) and ORs SF_ST_TIMEOUT into *status (device,
+   required).  The kernel then exits normally; nothing faults or traps. */
+sf_status sf_selftest_bounded_wait(uint64_t limit_ns, uint32_t* status, cudaStream_t stream);
+
 /*
  * sf_frontier - Sec. 3 Eq. 1 on every step.
  *   d         [T][R][S] durations (device, 16-byte aligned).

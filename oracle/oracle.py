@@ -76,6 +76,8 @@ def lib():
         L.sfo_label_windows.argtypes = [_P, _I, _I, _I, _I, _P, _P, _P, ctypes.c_int32,
                                         ctypes.POINTER(Config), _P, _P, _P, _P, _P, _P, _P, _P, _P,
                                         _P, _P]
+        L.sfo_baselines.argtypes = [_P, _I, _I, _I, _I, _I, _P, _P, _P, _P]
+        L.sfo_baselines.restype = ctypes.c_int
         L.sfo_config_default.argtypes = [ctypes.POINTER(Config)]
         for f in ("sfo_frontier", "sfo_windows", "sfo_topk", "sfo_window_median", "sfo_direct_gain",
                   "sfo_label_windows"):
@@ -229,3 +231,26 @@ def label_windows(d, W: int, role=None, missing=None, wall=None, other_stage: in
                                    _ptr(out.gain), _ptr(out.X), _ptr(out.D), _ptr(out.Y),
                                    _ptr(out.m), _ptr(out.n_confident), _ptr(out.n_switch)))
     return out
+
+
+@dataclass
+class Baselines:
+    M: np.ndarray      # [nW][S] sum_t max_r d
+    SUM: np.ndarray    # [nW][S] sum_t sum_r d (Python ints, exact)
+    SLOW: np.ndarray   # [nW][S] slowest-rank breakdown
+    RANK0: np.ndarray  # [nW][S] rank-0 local total
+
+
+def baselines(d, W: int, t0: int = 0) -> Baselines:
+    """Routing baselines of Sec. 3 (per-stage max / average) and Sec. 6."""
+    d = _d(d)
+    T, R, S = d.shape
+    nW = num_windows(t0, T, W)
+    M = np.empty((nW, S), np.int64)
+    SUM = np.empty((nW, S, 2), np.uint64)
+    SLOW = np.empty((nW, S), np.int64)
+    R0 = np.empty((nW, S), np.int64)
+    _check(lib().sfo_baselines(_ptr(d), T, R, S, t0, W, _ptr(M), _ptr(SUM), _ptr(SLOW), _ptr(R0)))
+    total = np.array([[int(SUM[w, s, 1]) << 64 | int(SUM[w, s, 0]) for s in range(S)] for w in range(nW)],
+                     dtype=object)
+    return Baselines(M, total, SLOW, R0)

@@ -390,3 +390,49 @@ int sfo_label_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t
   free(P);
   return rc;
 }
+
+int sfo_baselines(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W, int64_t* M,
+                  uint64_t* SUM, int64_t* SLOW, int64_t* RANK0) {
+  if (!d || !check_shape(T, R, S) || W < 1 || W > 65536 || t0 < 0) return SFO_BADARG;
+  int64_t w_first = t0 / W;
+  int64_t nW = (t0 + T - 1) / W - w_first + 1;
+  if (M) memset(M, 0, sizeof(int64_t) * (size_t)(nW * S));
+  if (SUM) memset(SUM, 0, sizeof(uint64_t) * (size_t)(nW * S * 2));
+  if (SLOW) memset(SLOW, 0, sizeof(int64_t) * (size_t)(nW * S));
+  if (RANK0) memset(RANK0, 0, sizeof(int64_t) * (size_t)(nW * S));
+  for (int64_t t = 0; t < T; ++t) {
+    const int64_t* dt = d + t * R * S;
+    int64_t w = (t0 + t) / W - w_first;
+    /* the slowest rank: largest total, lowest rank on ties */
+    int64_t slow = 0, best = -1;
+    for (int64_t r = 0; r < R; ++r) {
+      int64_t tot = 0;
+      for (int64_t s = 0; s < S; ++s) {
+        int64_t v = dt[r * S + s];
+        if (v < 0) return SFO_NEGATIVE;
+        if (v >= LIMIT47) return SFO_RANGE;
+        tot += v;
+      }
+      if (tot >= LIMIT47) return SFO_RANGE;
+      if (tot > best) { best = tot; slow = r; }
+    }
+    for (int64_t s = 0; s < S; ++s) {
+      int64_t mx = dt[s];
+      unsigned __int128 sum = 0;
+      for (int64_t r = 0; r < R; ++r) {
+        if (dt[r * S + s] > mx) mx = dt[r * S + s];
+        sum += (unsigned __int128)dt[r * S + s];
+      }
+      if (M) M[w * S + s] += mx;
+      if (SUM) {
+        unsigned __int128 acc = ((unsigned __int128)SUM[(w * S + s) * 2 + 1] << 64) | SUM[(w * S + s) * 2];
+        acc += sum;
+        SUM[(w * S + s) * 2] = (uint64_t)acc;
+        SUM[(w * S + s) * 2 + 1] = (uint64_t)(acc >> 64);
+      }
+      if (SLOW) SLOW[w * S + s] += dt[slow * S + s];
+      if (RANK0) RANK0[w * S + s] += dt[s];
+    }
+  }
+  return SFO_OK;
+}

@@ -83,6 +83,17 @@ int sfo_label_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t
                       int64_t* X, int64_t* D, int64_t* Y, int64_t* m, int32_t* n_confident,
                       int32_t* n_switch);
 
+/* Routing baselines the paper compares against (Sec. 3 per-stage max and
+   average; Sec. 6 routing table), per window and stage:
+     M    = sum_t max_r d[t,r,s]                      (per-stage max)
+     SUM  = sum_t sum_r d[t,r,s], as 128 bits (lo,hi)  (per-stage average x R)
+     SLOW = sum_t d[t,r*_t,s], r*_t the lowest rank with the largest total
+            (slowest-rank breakdown)
+     RANK0= sum_t d[t,0,s]                            (rank-0 local total)
+   Windows as in sfo_windows (t0, W).  Outputs overwritten; each nullable. */
+int sfo_baselines(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W, int64_t* M,
+                  uint64_t* SUM, int64_t* SLOW, int64_t* RANK0);
+
 void sfo_config_default(sfo_config* cfg);
 
 #ifdef __cplusplus

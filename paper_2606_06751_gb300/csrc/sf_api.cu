@@ -5,6 +5,7 @@
 #include <atomic>
 #include <cstring>
 
+#include "sf_device.cuh"
 #include "sf_launch.h"
 #include "stagefrontier.h"
 
@@ -265,6 +266,12 @@ sf_status sf_label_gates(int64_t T, int64_t R, int64_t S, int64_t W, const int64
   g.n_confident = n_confident;
   g.n_switch = n_switch;
   return cuda_status(launch_gates(g, stream));
+}
+
+sf_status sf_selftest_bounded_wait(uint64_t limit_ns, uint32_t* status, cudaStream_t stream) {
+  if (!status || limit_ns == 0 || limit_ns > kWaitLimitNs) return SF_EINVAL;
+  if (!aligned(status, 4)) return SF_EINVAL_ALIGN;
+  return cuda_status(launch_wait_selftest(limit_ns, status, stream));
 }
 
 size_t sf_label_windows_workspace_size(int64_t T, int64_t R, int64_t S, int64_t W) {

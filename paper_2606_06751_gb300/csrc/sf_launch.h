@@ -47,6 +47,7 @@ int sm_count();                     // SMs of the current device (cached)
 void count_launch(uint64_t n = 1);  // bump the library's launch counter
 
 cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t stream);
+cudaError_t launch_wait_selftest(uint64_t limit_ns, uint32_t* status, cudaStream_t stream);
 cudaError_t launch_stream_pass(const StreamJob& job, cudaStream_t stream);
 cudaError_t launch_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W,
                                  int64_t* m, uint32_t* status, cudaStream_t stream);

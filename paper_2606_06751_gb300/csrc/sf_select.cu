@@ -655,7 +655,30 @@ cudaError_t launch_median_tma(const CUtensorMap& map, int64_t T, int64_t RS, int
   return cudaGetLastError();
 }
 
+// Self-test of the bounded wait: every thread waits on an mbarrier phase
+// that nothing completes (count 2, one arrival), so the wait must give up
+// after limit_ns, record SF_ST_TIMEOUT and let the kernel finish.
+__global__ void wait_selftest_kernel(uint64_t limit_ns, uint32_t* status) {
+  __shared__ uint64_t bar;
+  __shared__ int abort;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 2);
+    abort = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) mbar_arrive(&bar);  // one of the two arrivals the phase needs
+  const bool ok = mbar_wait_bounded(&bar, 0, &abort, limit_ns);
+  if (threadIdx.x == 0) report(status, ok ? 0u : SF_ST_TIMEOUT);
+}
+
 }  // namespace
+
+cudaError_t launch_wait_selftest(uint64_t limit_ns, uint32_t* status, cudaStream_t stream) {
+  count_launch();
+  wait_selftest_kernel<<<1, 64, 0, stream>>>(limit_ns, status);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t stream) {
   if (bytes == 0) return cudaSuccess;

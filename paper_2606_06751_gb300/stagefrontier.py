@@ -72,6 +72,8 @@ def _load():
     L.sf_status_str.restype = ctypes.c_char_p
     L.sf_num_windows.argtypes = [I, I, I]
     L.sf_num_windows.restype = I
+    L.sf_selftest_bounded_wait.argtypes = [ctypes.c_uint64, P, S]
+    L.sf_selftest_bounded_wait.restype = ctypes.c_int
     L.sf_launch_count.argtypes = []
     L.sf_launch_count.restype = ctypes.c_uint64
     L.sf_label_config_default.argtypes = [ctypes.POINTER(LabelConfig)]
@@ -377,3 +379,7 @@ def sf_stream_windows(h_d: torch.Tensor, W: int, k: int, chunk_steps: int, bufs:
                                   _p(o.top_pair_value), _p(o.labels), _p(o.route_mask), _p(o.amb_mask), _p(o.share),
                                   _p(o.gain), _p(status), _stream(stream), cs.cuda_stream), "sf_stream_windows")
     return o
+
+
+def sf_selftest_bounded_wait(limit_ns: int, status: torch.Tensor, stream=None):
+    _check(_lib.sf_selftest_bounded_wait(limit_ns, _p(status), _stream(stream)), "sf_selftest_bounded_wait")

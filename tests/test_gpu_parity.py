@@ -280,3 +280,15 @@ def test_deterministic_repeat(sf):
     b = sf.sf_window_aggregate(d, 50)
     for name in ("X", "D", "E", "C", "step_lead"):
         assert torch.equal(getattr(a, name), getattr(b, name))
+
+
+def test_bounded_wait_times_out_cleanly(sf):
+    """A device wait that can never complete gives up after its limit, reports
+    SF_ST_TIMEOUT through the status word, and leaves the context usable."""
+    st = sf.new_status("cuda")
+    sf.sf_selftest_bounded_wait(50_000_000, st)      # 50 ms
+    torch.cuda.synchronize()
+    assert int(st.item()) == sf.SF_ST_TIMEOUT
+    d = dev(make(40, 64, 8, 1, "lognormal"))          # the context still runs work
+    f = sf.sf_frontier(d)
+    assert np.array_equal(host(f.a), O.frontier(host(d)).a)

@@ -407,3 +407,56 @@ def test_label_partial_last_window():
     # last window: 3 identical steps, three-way share tie, no confident leader
     assert L.labels[1] == O.L_FRONTIER_ACCOUNTING | O.L_CO_CRITICAL
     assert L.amb_mask[1] == 0b111 and L.n_confident[1] == 0
+
+
+# ---------------------------------------------------------------- routing baselines (Sec. 3, Sec. 6)
+
+@pytest.mark.parametrize("seed", range(3))
+def test_baselines_bounds_and_identities(seed):
+    """Props 1-2 summed over a window: D <= sum_s M <= min(R,S) D and
+    D <= sum_s SUM <= R D; the slowest rank's breakdown sums to D exactly (its
+    total is the makespan); rank 0's total never exceeds D."""
+    rng = np.random.default_rng(500 + seed)
+    T, R, S, W = 45, 7, 5, 10
+    d = rand_d(rng, T, R, S, hi=1000, zero_frac=0.2)
+    b = O.baselines(d, W)
+    w = O.windows(d, W)
+    for i in range(len(w.D)):
+        Dw = int(w.D[i])
+        assert Dw <= int(b.M[i].sum()) <= min(R, S) * Dw
+        assert Dw <= sum(b.SUM[i]) <= R * Dw
+        assert int(b.SLOW[i].sum()) == Dw
+        assert int(b.RANK0[i].sum()) <= Dw
+    # against numpy reductions of the same definitions
+    lead = O.frontier(d).lead[:, -1]
+    for i in range(len(w.D)):
+        blk = slice(i * W, (i + 1) * W)
+        assert (b.M[i] == d[blk].max(axis=1).sum(axis=0)).all()
+        assert list(b.SUM[i]) == [int(x) for x in d[blk].sum(axis=(0, 1))]
+        assert (b.SLOW[i] == d[blk][np.arange(d[blk].shape[0]), lead[blk]].sum(axis=0)).all()
+        assert (b.RANK0[i] == d[blk, 0, :].sum(axis=0)).all()
+
+
+def test_baselines_special_cases():
+    rng = np.random.default_rng(9)
+    one = rand_d(rng, 12, 1, 4)
+    b, w = O.baselines(one, 5), O.windows(one, 5)
+    for arr in (b.M, b.SLOW, b.RANK0):                 # R = 1: every summary is the accounting
+        assert (arr == w.X).all()
+    base = rand_d(rng, 12, 1, 4)
+    same = np.repeat(base, 6, axis=1)                  # identical ranks
+    b, w = O.baselines(same, 5), O.windows(same, 5)
+    assert (b.M == w.X).all() and (b.SLOW == w.X).all()
+    assert [list(r) for r in b.SUM] == [[6 * int(x) for x in row] for row in w.X]
+    # Prop 1 tightness: min(R,S) pairs of duration Dv, no rank holding two
+    dt = np.zeros((1, 3, 5), np.int64)
+    for i in range(3):
+        dt[0, i, i] = 7
+    b, w = O.baselines(dt, 1), O.windows(dt, 1)
+    assert b.M[0].sum() == 3 * w.D[0]
+
+
+def test_baselines_big_sums_are_exact():
+    d = np.full((4, 3, 1), (1 << 46) + 12345, np.int64)  # each rank total just under 2^47
+    b = O.baselines(d, 4)
+    assert b.SUM[0][0] == 12 * ((1 << 46) + 12345)    # above 2^49, exact
