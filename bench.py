@@ -227,6 +227,8 @@ class Pipeline:
                              e((nW,), torch.int32))
         self.win = sf.Windows(e((nW, S), torch.int64), e((nW,), torch.int64), e((nW, S, R), torch.int64),
                               e((nW, S, R), torch.int32), e((T,), torch.uint8))
+        self.base = sf.Baselines(e((nW, S), torch.int64), e((nW, S, 2), torch.uint64), e((nW, S), torch.int64),
+                                 e((nW, S), torch.int64))
         self.status = sf.new_status(dev)
         self.names = ["window_median", "direct_gain", "topk_suspects", "label_gates"]
         self.events = None
@@ -257,6 +259,10 @@ class Pipeline:
         self.sf.sf_window_aggregate(self.d, self.w.W, X=self.win.X, D=self.win.D, E=self.win.E, C=self.win.C,
                                     step_lead=self.win.step_lead, status=self.status)
 
+    def baselines(self):
+        """The routing-baseline pass (sf_window_baselines)."""
+        self.sf.sf_window_baselines(self.d, self.w.W, out=self.base, status=self.status)
+
     def results(self):
         return [self.lab.labels, self.lab.route_mask, self.lab.amb_mask, self.lab.share, self.lab.gain,
                 self.top.stage, self.top.pair, self.top.pair_value, self.ev.X, self.ev.D]
@@ -270,6 +276,7 @@ class Pipeline:
             "topk_suspects": nW * w.S * (w.R + 1) * 8 + nW * w.k * 24,
             "label_gates": nW * (2 * w.S + 1) * 8 + w.T + nW * (3 * 4 + 2 * w.S * 8),
             "window_aggregate": din + nW * w.S * (w.R * 12 + 8) + nW * 8 + w.T,
+            "window_baselines": din + nW * w.S * 40 + w.T * w.S * 16,
         }
 
 
@@ -315,8 +322,9 @@ def run_ours(args):
     achieved = algo[dominant] / avg[dominant] / 1e9
     value = records * ws * args.steps / secs
 
-    # the standalone frontier/aggregation pass, timed on its own
+    # the standalone frontier/aggregation pass and the routing-baseline pass, each timed on its own
     agg_secs = timed_loop(pipe.aggregate, args.steps, args.warmup, ws, device, True) / args.steps
+    base_secs = timed_loop(pipe.baselines, args.steps, args.warmup, ws, device, True) / args.steps
 
     # end to end through the host-memory entry point: every step streams the
     # pinned host tensor to the GPU in 2000-step chunks (copies overlapping the
@@ -365,6 +373,9 @@ def run_ours(args):
         "frontier_pass": {"entry": "sf_window_aggregate", "ms": round(agg_secs * 1e3, 4),
                           "gbs": round(agg_gbs, 1), "frac": round(agg_gbs / peak, 4),
                           "records_per_s": records / agg_secs},
+        "baselines_pass": {"entry": "sf_window_baselines", "ms": round(base_secs * 1e3, 4),
+                           "gbs": round(algo["window_baselines"] / base_secs / 1e9, 1),
+                           "frac": round(algo["window_baselines"] / base_secs / 1e9 / peak, 4)},
         "gpu_launches": int(launches * args.steps // (args.steps + args.warmup)),
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": w.nbytes, "d2h_bytes_per_step": d2h,
                 "entry": "sf_stream_windows", "chunk_steps": chunk},

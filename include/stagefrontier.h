@@ -120,6 +120,23 @@ sf_status sf_window_aggregate(const int64_t* d, int64_t T, int64_t R, int64_t S,
                               cudaStream_t stream);
 
 /*
+ * sf_window_baselines - the routing baselines the paper compares frontier
+ * accounting against (Sec. 3 per-stage max and average, Props 1-2; Sec. 6
+ * routing table), per window and stage, in one pass over d:
+ *   M     [nW][S]    sum_t max_r d[t,r,s]                  (per-stage max)
+ *   SUM   [nW][S][2] sum_t sum_r d[t,r,s] as a 128-bit (lo, hi) pair
+ *                    (per-stage average times R; exact)
+ *   SLOW  [nW][S]    sum_t d[t,r*,s], r* the step's slowest rank (largest total,
+ *                    lowest rank on ties): the slowest-rank breakdown
+ *   RANK0 [nW][S]    sum_t d[t,0,s]                          (rank-0 local total)
+ * Windows, t0 and accumulate as in sf_window_aggregate; all outputs device,
+ * required.
+ */
+sf_status sf_window_baselines(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W,
+                              int64_t* M, uint64_t* SUM, int64_t* SLOW, int64_t* RANK0,
+                              int32_t accumulate, uint32_t* status, cudaStream_t stream);
+
+/*
  * sf_topk_suspects - per window, the k stages with the largest X (Sec. 4
  * routing uses the top two shares) and the k (stage, rank) pairs with the
  * largest lead-rank credit E.  Order: value descending, then lower stage,

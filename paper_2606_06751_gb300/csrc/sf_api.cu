@@ -167,6 +167,39 @@ sf_status sf_window_aggregate(const int64_t* d, int64_t T, int64_t R, int64_t S,
   return cuda_status(launch_stream_pass(j, stream));
 }
 
+sf_status sf_window_baselines(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W,
+                              int64_t* M, uint64_t* SUM, int64_t* SLOW, int64_t* RANK0, int32_t accumulate,
+                              uint32_t* status, cudaStream_t stream) {
+  if (!d || !M || !SUM || !SLOW || !RANK0 || !shape_ok(T, R, S) || t0 < 0 || W < 1 || W > 65536 ||
+      (accumulate != 0 && accumulate != 1) || t0 > (int64_t(1) << 62) - T)
+    return SF_EINVAL;
+  if (!aligned(d, 16) || !aligned(M, 8) || !aligned(SUM, 8) || !aligned(SLOW, 8) || !aligned(RANK0, 8) ||
+      !aligned(status, 4))
+    return SF_EINVAL_ALIGN;
+  const int64_t nW = sf_num_windows(t0, T, W);
+  if (!accumulate) {
+    cudaError_t e = launch_zero(M, size_t(nW) * S * 8, stream);
+    if (e == cudaSuccess) e = launch_zero(SUM, size_t(nW) * S * 16, stream);
+    if (e == cudaSuccess) e = launch_zero(SLOW, size_t(nW) * S * 8, stream);
+    if (e == cudaSuccess) e = launch_zero(RANK0, size_t(nW) * S * 8, stream);
+    if (e != cudaSuccess) return SF_ECUDA;
+  }
+  StreamJob j;
+  j.d = d;
+  j.T = T;
+  j.R = R;
+  j.S = S;
+  j.t0 = t0;
+  j.W = W;
+  j.base = true;
+  j.bM = M;
+  j.bSUM = SUM;
+  j.bSLOW = SLOW;
+  j.bRANK0 = RANK0;
+  j.status = status;
+  return cuda_status(launch_stream_pass(j, stream));
+}
+
 sf_status sf_topk_suspects(const int64_t* X, const int64_t* E, int64_t nW, int64_t S, int64_t R, int32_t k,
                            int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair,
                            int64_t* top_pair_value, cudaStream_t stream) {

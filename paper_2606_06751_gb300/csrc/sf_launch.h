@@ -34,6 +34,12 @@ struct StreamJob {
   int64_t* Y = nullptr;
   uint64_t* quality = nullptr;
   uint32_t* status = nullptr;
+  // routing-baseline pass (sf_window_baselines)
+  bool base = false;
+  int64_t* bM = nullptr;
+  uint64_t* bSUM = nullptr;
+  int64_t* bSLOW = nullptr;
+  int64_t* bRANK0 = nullptr;
 };
 
 // cuTensorMapEncodeTiled from the driver, resolved once (null if unavailable).

@@ -51,7 +51,8 @@ constexpr int kR1MaxRows = kR1StageBytes / kRowBytes;   // 256 rows (the TMA box
 // holds a d tile in its first half and the matching m tile in its second.
 constexpr int kR1GainMaxRows = kR1MaxRows / 2;
 constexpr int kMaxStages = kR0Stages;
-constexpr int kRedSlots = 2 * kConsumerWarps * 32;    // double-buffered per-warp partials
+constexpr int kRedPerWarp = 64;                       // per-warp partials of one step (<= 2S + 1)
+constexpr int kRedSlots = 2 * kConsumerWarps * kRedPerWarp;  // double-buffered
 constexpr size_t kSmemBytes = 1024 /*alignment slack*/ + size_t(kRingBytes) +
                               2 * kMaxStages * sizeof(uint64_t) + 16 + kRedSlots * sizeof(uint64_t);
 
@@ -77,6 +78,12 @@ struct Params {
   uint64_t* quality;
   uint32_t* status;
   int m_by_tma;  // evidence pass, regime 1: m tiles arrive through the ring
+  // routing-baseline pass
+  const int64_t* d;
+  int64_t* bM;
+  uint64_t* bSUM;
+  int64_t* bSLOW;
+  int64_t* bRANK0;
 };
 
 __device__ __forceinline__ uint32_t hi32(int64_t v) {
@@ -181,6 +188,52 @@ __device__ __forceinline__ void finalize_gain(const Params& p, int S, int64_t t,
       atomicAdd(reinterpret_cast<unsigned long long*>(&p.E[idx]), static_cast<unsigned long long>(a));
     if (p.C) atomicAdd(&p.C[idx], 1);
   }
+}
+
+// Routing-baseline window accumulators (lane s: stage s).
+struct BaseAcc {
+  int64_t cur = -1;
+  int64_t m = 0, slow = 0, r0 = 0;
+  unsigned __int128 sum = 0;
+};
+
+__device__ __forceinline__ void flush_base(const Params& p, int S, BaseAcc& acc, int lane) {
+  if (acc.cur >= 0 && lane < S) {
+    const int64_t i = acc.cur * S + lane;
+    if (acc.m) atomicAdd(reinterpret_cast<unsigned long long*>(&p.bM[i]), static_cast<unsigned long long>(acc.m));
+    if (acc.sum) atomic_add_u128(p.bSUM + 2 * i, acc.sum);
+    if (acc.slow)
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.bSLOW[i]), static_cast<unsigned long long>(acc.slow));
+    if (acc.r0) atomicAdd(reinterpret_cast<unsigned long long*>(&p.bRANK0[i]), static_cast<unsigned long long>(acc.r0));
+  }
+  acc.m = acc.slow = acc.r0 = 0;
+  acc.sum = 0;
+}
+
+// Baseline epilogue for step t.  Lane s < S holds max_r d[t,r,s] and
+// sum_r d[t,r,s]; every lane holds the packed key of the slowest rank
+// (largest total, lowest rank on ties), whose row and rank 0's row are read
+// back from d (the step was just streamed, so these hit L2).
+__device__ __forceinline__ void finalize_base(const Params& p, int S, int64_t t, uint64_t mx, uint64_t sm,
+                                              uint64_t slowkey, int lane, BaseAcc& acc) {
+  const int64_t w = (p.t0 + t) / p.W - p.w_first;
+  if (w != acc.cur) {
+    flush_base(p, S, acc, lane);
+    acc.cur = w;
+  }
+  const int64_t rs = 65535 - static_cast<int64_t>(slowkey & 0xffffu);
+  if (lane < S && rs >= 0 && rs < p.R) {  // always in range for valid input
+    acc.m += static_cast<int64_t>(mx);
+    acc.sum += sm;
+    acc.slow += __ldg(p.d + (t * p.R + rs) * S + lane);
+    acc.r0 += __ldg(p.d + t * p.R * S + lane);
+  }
+}
+
+__device__ __forceinline__ uint64_t warp_sum_u64(uint64_t v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+  return v;
 }
 
 // Telemetry-quality sums of one thread (App. A closure / overlap), flushed per window.
@@ -357,6 +410,35 @@ struct GainRows {
   }
 };
 
+// Routing-baseline maxima and sums over the rank rows a thread visits.
+template <int S>
+struct BaseRows {
+  int64_t mx[S];
+  uint64_t sm[S];
+  uint64_t slow;  // (P_S << 16) | (65535 - r), max
+  __device__ __forceinline__ void init() {
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      mx[s] = 0;
+      sm[s] = 0;
+    }
+    slow = 0;
+  }
+  __device__ __forceinline__ void row(const int64_t (&v)[S], int32_t r, uint32_t& dor, uint32_t& tor) {
+    int64_t P = 0;
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      dor |= hi32(v[s]);
+      P += v[s];
+      mx[s] = v[s] > mx[s] ? v[s] : mx[s];
+      sm[s] += static_cast<uint64_t>(v[s]);
+    }
+    tor |= hi32(P);
+    const uint64_t k = (static_cast<uint64_t>(P) << 16) | static_cast<uint64_t>(65535 - r);
+    slow = k > slow ? k : slow;
+  }
+};
+
 template <int S>
 __device__ __forceinline__ int64_t pick(const int64_t (&v)[S], int idx) {
   int64_t o = 0;
@@ -449,13 +531,15 @@ __device__ void produce(const CUtensorMap* map, const CUtensorMap* map_m, const 
 }
 
 // --------------------------------------------------------------------------
-template <int S, bool GAIN>
+// MODE 0: frontier (+ window aggregation); 1: evidence pass; 2: routing baselines.
+template <int S, int MODE>
 __global__ void __launch_bounds__(kBlockThreads, 1)
     stream_kernel(const __grid_constant__ CUtensorMap map, const __grid_constant__ CUtensorMap map_m,
                   const Params p) {
+  constexpr bool GAIN = MODE == 1;
+  constexpr bool BASE = MODE == 2;
   constexpr bool kSwz = (S == 4 || S == 8 || S == 16);
   constexpr int U = S <= 8 ? 4 : 2;  // rank rows in flight per thread
-  constexpr int NV = GAIN ? 2 * S : S;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* ring = align_1024(smem_raw);
   uint64_t* full = reinterpret_cast<uint64_t*>(ring + kRingBytes);
@@ -485,6 +569,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
   uint32_t dor = 0, tor = 0;  // OR of duration / rank-total high words
   WinAcc acc;
   QualAcc qa;
+  BaseAcc bacc;
   const int R = static_cast<int>(p.R);
 
   if (p.regime == 0) {
@@ -502,7 +587,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
         const int64_t w = GAIN ? t / p.W : 0;
         if (GAIN && p.quality) qual_window(p, qa, w, lane);
         const int q0 = kk * R;
-        if constexpr (!GAIN) {
+        if constexpr (MODE == 0) {
           FrontierRows<S> rs;
           rs.init();
           if (have) {
@@ -523,6 +608,31 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
             if (lane == s) mykey = km;
           }
           finalize_frontier(p, S, t, mykey, lane, acc);
+        } else if constexpr (BASE) {
+          BaseRows<S> rs;
+          rs.init();
+          if (have) {
+            for (int r0 = lane; r0 < R; r0 += 32 * U) {
+              int64_t v[U][S];
+#pragma unroll
+              for (int u = 0; u < U; ++u)
+                if (r0 + 32 * u < R) load_row<S, kSwz>(tile, q0 + r0 + 32 * u, v[u]);
+#pragma unroll
+              for (int u = 0; u < U; ++u)
+                if (r0 + 32 * u < R) rs.row(v[u], r0 + 32 * u, dor, tor);
+            }
+          }
+          uint64_t myM = 0, mySum = 0;
+#pragma unroll
+          for (int s = 0; s < S; ++s) {
+            const uint64_t mx = warp_max_u64(static_cast<uint64_t>(rs.mx[s]));
+            const uint64_t sm = warp_sum_u64(rs.sm[s]);
+            if (lane == s) {
+              myM = mx;
+              mySum = sm;
+            }
+          }
+          finalize_base(p, S, t, myM, mySum, warp_max_u64(rs.slow), lane, bacc);
         } else {
           GainRows<S> rs;
           rs.init();
@@ -563,7 +673,10 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
       if (GAIN && p.quality) qual_window(p, qa, w, lane);
       FrontierRows<S> fr;
       GainRows<S> gr;
-      if constexpr (GAIN) gr.init(); else fr.init();
+      BaseRows<S> br;
+      if constexpr (GAIN) gr.init();
+      else if constexpr (BASE) br.init();
+      else fr.init();
       for (int k = 0; k < p.tiles_per_step; ++k, ++j) {
         const uint32_t st = j % kR1Stages, ph = (j / kR1Stages) & 1u;
         const bool have = mbar_wait_bounded(&full[st], ph, abort);
@@ -582,7 +695,10 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
                   load_row<S, kSwz>(tile, r0 + kConsumerThreads * u - rank_tile0, v[u]);
 #pragma unroll
               for (int u = 0; u < U; ++u)
-                if (r0 + kConsumerThreads * u < rank_end) fr.row(v[u], r0 + kConsumerThreads * u, dor, tor);
+                if (r0 + kConsumerThreads * u < rank_end) {
+                  if constexpr (BASE) br.row(v[u], r0 + kConsumerThreads * u, dor, tor);
+                  else fr.row(v[u], r0 + kConsumerThreads * u, dor, tor);
+                }
             }
           } else {
             for (int r = rank_fresh + ctid; r < rank_end; r += kConsumerThreads) {
@@ -599,12 +715,21 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
         if (lane == 0) mbar_arrive(&empty[st]);
       }
       // cross-rank reduction: warp redux, then one exchange through shared memory
-      uint64_t* slot = red + (buf * kConsumerWarps + warp) * 32;
+      uint64_t* slot = red + (buf * kConsumerWarps + warp) * kRedPerWarp;
+      uint64_t bslow = 0;
+      if constexpr (BASE) bslow = warp_max_u64(br.slow);
 #pragma unroll
       for (int s = 0; s < S; ++s) {
-        if constexpr (!GAIN) {
+        if constexpr (MODE == 0) {
           const uint64_t km = warp_max_u64(fr.key(s));
           if (lane == s) slot[s] = km;
+        } else if constexpr (BASE) {
+          const uint64_t mx = warp_max_u64(static_cast<uint64_t>(br.mx[s]));
+          const uint64_t sm = warp_sum_u64(br.sm[s]);
+          if (lane == s) {
+            slot[s] = mx;
+            slot[S + s] = sm;
+          }
         } else {
           const uint64_t f = warp_max_u64(gr.key(s));
           const uint64_t g = warp_max_u64(gr.G(s));
@@ -614,26 +739,35 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
           }
         }
       }
+      if (BASE && lane == 0) slot[2 * S] = bslow;
       named_barrier(1, kConsumerThreads);
       if (warp == 0) {
-        uint64_t v0 = 0, v1 = 0;
+        uint64_t v0 = 0, v1 = 0, v2 = 0;
         if (lane < S) {
 #pragma unroll
           for (int ww = 0; ww < kConsumerWarps; ++ww) {
-            const uint64_t* sl = red + (buf * kConsumerWarps + ww) * 32;
+            const uint64_t* sl = red + (buf * kConsumerWarps + ww) * kRedPerWarp;
             v0 = sl[lane] > v0 ? sl[lane] : v0;
             if (GAIN) v1 = sl[S + lane] > v1 ? sl[S + lane] : v1;
+            if (BASE) v1 += sl[S + lane];
           }
         }
-        if constexpr (!GAIN) finalize_frontier(p, S, t, v0, lane, acc);
+        if (BASE) {
+          for (int ww = 0; ww < kConsumerWarps; ++ww) {
+            const uint64_t k = red[(buf * kConsumerWarps + ww) * kRedPerWarp + 2 * S];
+            v2 = k > v2 ? k : v2;
+          }
+        }
+        if constexpr (MODE == 0) finalize_frontier(p, S, t, v0, lane, acc);
+        else if constexpr (BASE) finalize_base(p, S, t, v0, v1, v2, lane, bacc);
         else finalize_gain(p, S, t, v0, static_cast<int64_t>(v1), lane, acc);
       }
       buf ^= 1;
     }
-    (void)NV;
   }
 
-  if (p.X && (p.regime == 0 || warp == 0)) flush_window(p, S, acc, lane);
+  if (BASE && (p.regime == 0 || warp == 0)) flush_base(p, S, bacc, lane);
+  if (!BASE && p.X && (p.regime == 0 || warp == 0)) flush_window(p, S, acc, lane);
   if (GAIN && p.quality) qual_window(p, qa, -2, lane);
   const uint32_t bits = range_bits(__reduce_or_sync(kFull, dor), __reduce_or_sync(kFull, tor)) |
                         (*abort ? SF_ST_TIMEOUT : 0u);
@@ -644,10 +778,12 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
 // Generic path: any S <= 32, any R; one CTA of 256 threads per step range.
 constexpr int kGenThreads = 256;
 
-template <bool GAIN>
+template <int MODE>
 __global__ void __launch_bounds__(kGenThreads)
     stream_generic_kernel(const int64_t* __restrict__ d, const Params p) {
-  __shared__ uint64_t red[kGenThreads / 32][64];
+  constexpr bool GAIN = MODE == 1;
+  constexpr bool BASE = MODE == 2;
+  __shared__ uint64_t red[kGenThreads / 32][66];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int S = static_cast<int>(p.S);
   const int64_t R = p.R;
@@ -656,13 +792,15 @@ __global__ void __launch_bounds__(kGenThreads)
   uint32_t dor = 0, tor = 0;
   WinAcc acc;
   QualAcc qa;
+  BaseAcc bacc;
   for (int64_t t = t_begin; t < t_end; ++t) {
     const int64_t w = GAIN ? t / p.W : 0;
     if (GAIN && p.quality) qual_window(p, qa, w, lane);
     int64_t b0[32], b1[32];
     int32_t br[32];
+    uint64_t slow = 0;
     for (int s = 0; s < S; ++s) {
-      b0[s] = -1;
+      b0[s] = BASE ? 0 : -1;
       b1[s] = 0;
       br[s] = 0;
     }
@@ -674,12 +812,19 @@ __global__ void __launch_bounds__(kGenThreads)
         dor |= hi32(v);
         P += v;
         if (s == p.other_stage) other = v;
-        if (P > b0[s]) {
+        if (BASE) {
+          b0[s] = v > b0[s] ? v : b0[s];
+          b1[s] += v;
+        } else if (P > b0[s]) {
           b0[s] = P;
           br[s] = static_cast<int32_t>(r);
         }
       }
       tor |= hi32(P);
+      if (BASE) {
+        const uint64_t k = (static_cast<uint64_t>(P) << 16) | static_cast<uint64_t>(65535 - r);
+        slow = k > slow ? k : slow;
+      }
       if (GAIN) {
         const int64_t* mr = p.m + (w * R + r) * S;
         for (int s = 0; s < S; ++s) {
@@ -691,29 +836,41 @@ __global__ void __launch_bounds__(kGenThreads)
       }
     }
     for (int s = 0; s < S; ++s) {
-      const uint64_t k0 =
-          b0[s] < 0 ? 0ull : (static_cast<uint64_t>(b0[s]) << 16) | static_cast<uint64_t>(65535 - br[s]);
+      uint64_t k0;
+      if (BASE) k0 = static_cast<uint64_t>(b0[s]);
+      else k0 = b0[s] < 0 ? 0ull : (static_cast<uint64_t>(b0[s]) << 16) | static_cast<uint64_t>(65535 - br[s]);
       const uint64_t m0 = warp_max_u64(k0);
-      const uint64_t m1 = GAIN ? warp_max_u64(static_cast<uint64_t>(b1[s])) : 0;
+      const uint64_t m1 = GAIN   ? warp_max_u64(static_cast<uint64_t>(b1[s]))
+                          : BASE ? warp_sum_u64(static_cast<uint64_t>(b1[s]))
+                                 : 0;
       if (lane == 0) {
         red[warp][s] = m0;
         red[warp][32 + s] = m1;
       }
     }
+    if (BASE) {
+      const uint64_t ks = warp_max_u64(slow);
+      if (lane == 0) red[warp][64] = ks;
+    }
     __syncthreads();
     if (warp == 0) {
-      uint64_t v0 = 0, v1 = 0;
+      uint64_t v0 = 0, v1 = 0, v2 = 0;
       if (lane < S)
         for (int ww = 0; ww < kGenThreads / 32; ++ww) {
           v0 = red[ww][lane] > v0 ? red[ww][lane] : v0;
-          v1 = red[ww][32 + lane] > v1 ? red[ww][32 + lane] : v1;
+          if (BASE) v1 += red[ww][32 + lane];
+          else v1 = red[ww][32 + lane] > v1 ? red[ww][32 + lane] : v1;
         }
+      if (BASE)
+        for (int ww = 0; ww < kGenThreads / 32; ++ww) v2 = red[ww][64] > v2 ? red[ww][64] : v2;
       if (GAIN) finalize_gain(p, S, t, v0, static_cast<int64_t>(v1), lane, acc);
+      else if (BASE) finalize_base(p, S, t, v0, v1, v2, lane, bacc);
       else finalize_frontier(p, S, t, v0, lane, acc);
     }
     __syncthreads();
   }
-  if (p.X && warp == 0) flush_window(p, S, acc, lane);
+  if (BASE && warp == 0) flush_base(p, S, bacc, lane);
+  if (!BASE && p.X && warp == 0) flush_window(p, S, acc, lane);
   if (GAIN && p.quality) qual_window(p, qa, -2, lane);
   const uint32_t bits = range_bits(__reduce_or_sync(kFull, dor), __reduce_or_sync(kFull, tor));
   if (lane == 0) report(p.status, bits);
@@ -721,20 +878,20 @@ __global__ void __launch_bounds__(kGenThreads)
 
 // --------------------------------------------------------------------------
 // Host side
-template <int S, bool GAIN>
+template <int S, int MODE>
 cudaError_t prepare_fast() {
-  return cudaFuncSetAttribute(stream_kernel<S, GAIN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  return cudaFuncSetAttribute(stream_kernel<S, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               static_cast<int>(kSmemBytes));
 }
 
-template <bool GAIN>
+template <int MODE>
 cudaError_t dispatch_fast(int S, const CUtensorMap& map, const CUtensorMap& map_m, const Params& p, int grid,
                           cudaStream_t stream) {
 #define SF_CASE(SV)                                                                          \
   case SV: {                                                                                 \
-    cudaError_t e = prepare_fast<SV, GAIN>();                                     \
+    cudaError_t e = prepare_fast<SV, MODE>();                                     \
     if (e != cudaSuccess) return e;                                                          \
-    stream_kernel<SV, GAIN><<<grid, kBlockThreads, kSmemBytes, stream>>>(map, map_m, p);     \
+    stream_kernel<SV, MODE><<<grid, kBlockThreads, kSmemBytes, stream>>>(map, map_m, p);     \
     return cudaGetLastError();                                                               \
   }
   switch (S) {
@@ -791,6 +948,11 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
   p.Y = j.Y;
   p.quality = j.quality;
   p.status = j.status;
+  p.d = j.d;
+  p.bM = j.bM;
+  p.bSUM = j.bSUM;
+  p.bSLOW = j.bSLOW;
+  p.bRANK0 = j.bRANK0;
 
   const int64_t RS = j.R * j.S;
   const int64_t step_rows = RS / 16;
@@ -846,13 +1008,15 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
     const int64_t units = p.regime == 0 ? (j.T + p.K - 1) / p.K : j.T;
     const int grid = static_cast<int>(std::min<int64_t>(sms, units));
     count_launch();
-    return j.gain ? dispatch_fast<true>(static_cast<int>(j.S), map, map_m, p, grid, stream)
-                  : dispatch_fast<false>(static_cast<int>(j.S), map, map_m, p, grid, stream);
+    if (j.base) return dispatch_fast<2>(static_cast<int>(j.S), map, map_m, p, grid, stream);
+    return j.gain ? dispatch_fast<1>(static_cast<int>(j.S), map, map_m, p, grid, stream)
+                  : dispatch_fast<0>(static_cast<int>(j.S), map, map_m, p, grid, stream);
   }
   const int grid = static_cast<int>(std::min<int64_t>(int64_t(sms) * 4, j.T));
   count_launch();
-  if (j.gain) stream_generic_kernel<true><<<grid, kGenThreads, 0, stream>>>(j.d, p);
-  else stream_generic_kernel<false><<<grid, kGenThreads, 0, stream>>>(j.d, p);
+  if (j.base) stream_generic_kernel<2><<<grid, kGenThreads, 0, stream>>>(j.d, p);
+  else if (j.gain) stream_generic_kernel<1><<<grid, kGenThreads, 0, stream>>>(j.d, p);
+  else stream_generic_kernel<0><<<grid, kGenThreads, 0, stream>>>(j.d, p);
   return cudaGetLastError();
 }
 

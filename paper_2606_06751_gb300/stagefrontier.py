@@ -53,6 +53,7 @@ def _load():
         "sf_frontier": [P, I, I, I, P, P, P, P, S],
         "sf_window_aggregate": [P, I, I, I, I, I, P, P, P, P, P, I32, P, S],
         "sf_topk_suspects": [P, P, I, I, I, I32, P, P, P, P, S],
+        "sf_window_baselines": [P, I, I, I, I, I, P, P, P, P, I32, P, S],
         "sf_window_median": [P, I, I, I, I, P, P, S],
         "sf_direct_gain": [P, I, I, I, I, P, P, I32, Ratio, P, P, P, P, P, P, P, P, S],
         "sf_label_gates": [I, I, I, I, P, P, P, P, P, P, P, ctypes.POINTER(LabelConfig), P, P, P, P,
@@ -383,3 +384,23 @@ def sf_stream_windows(h_d: torch.Tensor, W: int, k: int, chunk_steps: int, bufs:
 
 def sf_selftest_bounded_wait(limit_ns: int, status: torch.Tensor, stream=None):
     _check(_lib.sf_selftest_bounded_wait(limit_ns, _p(status), _stream(stream)), "sf_selftest_bounded_wait")
+
+
+@dataclass
+class Baselines:
+    M: torch.Tensor      # [nW][S] sum_t max_r d
+    SUM: torch.Tensor    # [nW][S][2] uint64 (lo, hi) of sum_t sum_r d
+    SLOW: torch.Tensor   # [nW][S] slowest-rank breakdown
+    RANK0: torch.Tensor  # [nW][S] rank-0 local total
+
+
+def sf_window_baselines(d, W: int, t0: int = 0, out: Optional[Baselines] = None, accumulate: bool = False,
+                        status=None, stream=None) -> Baselines:
+    T, R, S = _d3(d)
+    nW = num_windows(t0, T, W)
+    if out is None:
+        out = Baselines(_empty((nW, S), torch.int64, d), _empty((nW, S, 2), torch.uint64, d),
+                        _empty((nW, S), torch.int64, d), _empty((nW, S), torch.int64, d))
+    _check(_lib.sf_window_baselines(_p(d), T, R, S, t0, W, _p(out.M), _p(out.SUM), _p(out.SLOW), _p(out.RANK0),
+                                    1 if accumulate else 0, _p(status), _stream(stream)), "sf_window_baselines")
+    return out

@@ -292,3 +292,21 @@ def test_bounded_wait_times_out_cleanly(sf):
     d = dev(make(40, 64, 8, 1, "lognormal"))          # the context still runs work
     f = sf.sf_frontier(d)
     assert np.array_equal(host(f.a), O.frontier(host(d)).a)
+
+
+@pytest.mark.parametrize("T,R,S", SHAPES[:4] + SHAPES[5:9] + SHAPES[14:18] + [(3000, 512, 4), (200000, 8, 6)])
+@pytest.mark.parametrize("t0,W", [(0, 7), (13, 100)])
+def test_baselines_parity(sf, T, R, S, t0, W):
+    """Per-stage max, sum (128-bit), slowest-rank breakdown and rank-0 total
+    per window against the oracle, on every streaming path."""
+    d_np = make(T, R, S, T + 3 * R + S, "ties" if R < 100 else "lognormal")
+    o = O.baselines(d_np, W, t0)
+    st = sf.new_status("cuda")
+    b = sf.sf_window_baselines(dev(d_np), W, t0=t0, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert np.array_equal(host(b.M), o.M)
+    assert np.array_equal(host(b.SLOW), o.SLOW) and np.array_equal(host(b.RANK0), o.RANK0)
+    s2 = host(b.SUM)
+    got = [[int(s2[w, s, 1]) << 64 | int(s2[w, s, 0]) for s in range(S)] for w in range(s2.shape[0])]
+    assert got == [list(r) for r in o.SUM]
