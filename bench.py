@@ -229,6 +229,8 @@ class Pipeline:
                               e((nW, S, R), torch.int32), e((T,), torch.uint8))
         self.base = sf.Baselines(e((nW, S), torch.int64), e((nW, S, 2), torch.uint64), e((nW, S), torch.int64),
                                  e((nW, S), torch.int64))
+        self.lag = sf.Lag(e((T, S), torch.int64), e((T, S), torch.int64), e((T, S), torch.int64))
+        self.spread = e((nW, S), torch.int64)
         self.status = sf.new_status(dev)
         self.names = ["window_median", "direct_gain", "topk_suspects", "label_gates"]
         self.events = None
@@ -263,6 +265,14 @@ class Pipeline:
         """The routing-baseline pass (sf_window_baselines)."""
         self.sf.sf_window_baselines(self.d, self.w.W, out=self.base, status=self.status)
 
+    def rank_lag(self):
+        """The cross-rank lag / delta-lag / gap pass (sf_rank_lag)."""
+        self.sf.sf_rank_lag(self.d, out=self.lag, status=self.status)
+
+    def raw_spread(self):
+        """The raw rank spread per window (sf_raw_spread)."""
+        self.sf.sf_raw_spread(self.d, self.w.W, spread=self.spread, status=self.status)
+
     def results(self):
         return [self.lab.labels, self.lab.route_mask, self.lab.amb_mask, self.lab.share, self.lab.gain,
                 self.top.stage, self.top.pair, self.top.pair_value, self.ev.X, self.ev.D]
@@ -277,6 +287,8 @@ class Pipeline:
             "label_gates": nW * (2 * w.S + 1) * 8 + w.T + nW * (3 * 4 + 2 * w.S * 8),
             "window_aggregate": din + nW * w.S * (w.R * 12 + 8) + nW * 8 + w.T,
             "window_baselines": din + nW * w.S * 40 + w.T * w.S * 16,
+            "rank_lag": din + 3 * w.T * w.S * 8,
+            "raw_spread": din + nW * w.S * 8,
         }
 
 
@@ -325,6 +337,8 @@ def run_ours(args):
     # the standalone frontier/aggregation pass and the routing-baseline pass, each timed on its own
     agg_secs = timed_loop(pipe.aggregate, args.steps, args.warmup, ws, device, True) / args.steps
     base_secs = timed_loop(pipe.baselines, args.steps, args.warmup, ws, device, True) / args.steps
+    lag_secs = timed_loop(pipe.rank_lag, args.steps, args.warmup, ws, device, True) / args.steps
+    spread_secs = timed_loop(pipe.raw_spread, args.steps, args.warmup, ws, device, True) / args.steps
 
     # end to end through the host-memory entry point: every step streams the
     # pinned host tensor to the GPU in 2000-step chunks (copies overlapping the
@@ -376,6 +390,12 @@ def run_ours(args):
         "baselines_pass": {"entry": "sf_window_baselines", "ms": round(base_secs * 1e3, 4),
                            "gbs": round(algo["window_baselines"] / base_secs / 1e9, 1),
                            "frac": round(algo["window_baselines"] / base_secs / 1e9 / peak, 4)},
+        "lag_pass": {"entry": "sf_rank_lag", "ms": round(lag_secs * 1e3, 4),
+                     "gbs": round(algo["rank_lag"] / lag_secs / 1e9, 1),
+                     "frac": round(algo["rank_lag"] / lag_secs / 1e9 / peak, 4)},
+        "spread_pass": {"entry": "sf_raw_spread", "ms": round(spread_secs * 1e3, 4),
+                        "gbs": round(algo["raw_spread"] / spread_secs / 1e9, 1),
+                        "frac": round(algo["raw_spread"] / spread_secs / 1e9 / peak, 4)},
         "gpu_launches": int(launches * args.steps // (args.steps + args.warmup)),
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": w.nbytes, "d2h_bytes_per_step": d2h,
                 "entry": "sf_stream_windows", "chunk_steps": chunk},

@@ -137,6 +137,26 @@ sf_status sf_window_baselines(const int64_t* d, int64_t T, int64_t R, int64_t S,
                               int32_t accumulate, uint32_t* status, cudaStream_t stream);
 
 /*
+ * sf_rank_lag - localization evidence of Sec. 4 per step and stage:
+ *   L  [T][S] lag F[t,s] - median_r P[t,r,s] (lower median over ranks),
+ *   dL [T][S] its increment L[t,s] - L[t,s-1] (L[t,-1] = 0),
+ *   G  [T][S] max-minus-second-max gap F[t,s] - (second largest P[t,r,s]; a
+ *             tie at the top counts as the second, so ties give 0; R = 1 gives 0).
+ * Outputs device, nullable (at least one).
+ */
+sf_status sf_rank_lag(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t* L, int64_t* dL, int64_t* G,
+                      uint32_t* status, cudaStream_t stream);
+
+/*
+ * sf_raw_spread - the raw rank spread of the Sec. 6 routing table, per window
+ * and stage: sum_t (max_r d[t,r,s] - median_r d[t,r,s]), lower median over
+ * ranks.  spread [nW][S] device; windows, t0 and accumulate as in
+ * sf_window_aggregate.
+ */
+sf_status sf_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W,
+                        int64_t* spread, int32_t accumulate, uint32_t* status, cudaStream_t stream);
+
+/*
  * sf_topk_suspects - per window, the k stages with the largest X (Sec. 4
  * routing uses the top two shares) and the k (stage, rank) pairs with the
  * largest lead-rank credit E.  Order: value descending, then lower stage,

@@ -78,6 +78,10 @@ def lib():
                                         _P, _P]
         L.sfo_baselines.argtypes = [_P, _I, _I, _I, _I, _I, _P, _P, _P, _P]
         L.sfo_baselines.restype = ctypes.c_int
+        L.sfo_rank_lag.argtypes = [_P, _I, _I, _I, _P, _P, _P]
+        L.sfo_rank_lag.restype = ctypes.c_int
+        L.sfo_raw_spread.argtypes = [_P, _I, _I, _I, _I, _I, _P]
+        L.sfo_raw_spread.restype = ctypes.c_int
         L.sfo_config_default.argtypes = [ctypes.POINTER(Config)]
         for f in ("sfo_frontier", "sfo_windows", "sfo_topk", "sfo_window_median", "sfo_direct_gain",
                   "sfo_label_windows"):
@@ -254,3 +258,28 @@ def baselines(d, W: int, t0: int = 0) -> Baselines:
     total = np.array([[int(SUM[w, s, 1]) << 64 | int(SUM[w, s, 0]) for s in range(S)] for w in range(nW)],
                      dtype=object)
     return Baselines(M, total, SLOW, R0)
+
+
+@dataclass
+class Lag:
+    L: np.ndarray   # [T][S] F - median_r P
+    dL: np.ndarray  # [T][S] increment of L over stages
+    G: np.ndarray   # [T][S] max-minus-second-max gap
+
+
+def rank_lag(d) -> Lag:
+    """Sec. 4 localization evidence per step and stage."""
+    d = _d(d)
+    T, R, S = d.shape
+    out = Lag(np.empty((T, S), np.int64), np.empty((T, S), np.int64), np.empty((T, S), np.int64))
+    _check(lib().sfo_rank_lag(_ptr(d), T, R, S, _ptr(out.L), _ptr(out.dL), _ptr(out.G)))
+    return out
+
+
+def raw_spread(d, W: int, t0: int = 0) -> np.ndarray:
+    """Sec. 6 raw rank spread per window and stage."""
+    d = _d(d)
+    T, R, S = d.shape
+    out = np.empty((num_windows(t0, T, W), S), np.int64)
+    _check(lib().sfo_raw_spread(_ptr(d), T, R, S, t0, W, _ptr(out)))
+    return out

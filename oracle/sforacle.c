@@ -436,3 +436,61 @@ int sfo_baselines(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0,
   }
   return SFO_OK;
 }
+
+int sfo_rank_lag(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t* L, int64_t* dL, int64_t* G) {
+  if (!d || !check_shape(T, R, S)) return SFO_BADARG;
+  int64_t* P = (int64_t*)malloc(sizeof(int64_t) * (size_t)R);
+  int64_t* col = (int64_t*)malloc(sizeof(int64_t) * (size_t)R);
+  int rc = (P && col) ? SFO_OK : SFO_BADARG;
+  for (int64_t t = 0; t < T && rc == SFO_OK; ++t) {
+    for (int64_t r = 0; r < R; ++r) P[r] = 0;
+    int64_t prev = 0;
+    for (int64_t s = 0; s < S; ++s) {
+      for (int64_t r = 0; r < R; ++r) {
+        int64_t v = d[(t * R + r) * S + s];
+        if (v < 0) { rc = SFO_NEGATIVE; break; }
+        if (v >= LIMIT47) { rc = SFO_RANGE; break; }
+        P[r] += v;
+        col[r] = P[r];
+      }
+      if (rc != SFO_OK) break;
+      qsort(col, (size_t)R, sizeof(int64_t), cmp_i64);
+      const int64_t F = col[R - 1];                      /* F[t,s] = max_r P */
+      const int64_t med = col[(R - 1) / 2];              /* lower median over ranks */
+      const int64_t second = R >= 2 ? col[R - 2] : F;    /* second largest, ties counted */
+      const int64_t lag = F - med;
+      if (L) L[t * S + s] = lag;
+      if (dL) dL[t * S + s] = lag - prev;
+      if (G) G[t * S + s] = F - second;
+      prev = lag;
+    }
+    for (int64_t r = 0; r < R && rc == SFO_OK; ++r)
+      if (P[r] >= LIMIT47) rc = SFO_RANGE;
+  }
+  free(P);
+  free(col);
+  return rc;
+}
+
+int sfo_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W, int64_t* SPREAD) {
+  if (!d || !SPREAD || !check_shape(T, R, S) || W < 1 || W > 65536 || t0 < 0) return SFO_BADARG;
+  const int64_t w_first = t0 / W, nW = (t0 + T - 1) / W - w_first + 1;
+  memset(SPREAD, 0, sizeof(int64_t) * (size_t)(nW * S));
+  int64_t* col = (int64_t*)malloc(sizeof(int64_t) * (size_t)R);
+  if (!col) return SFO_BADARG;
+  int rc = SFO_OK;
+  for (int64_t t = 0; t < T && rc == SFO_OK; ++t) {
+    const int64_t w = (t0 + t) / W - w_first;
+    for (int64_t s = 0; s < S; ++s) {
+      for (int64_t r = 0; r < R; ++r) {
+        col[r] = d[(t * R + r) * S + s];
+        if (col[r] < 0) rc = SFO_NEGATIVE;
+        else if (col[r] >= LIMIT47) rc = SFO_RANGE;
+      }
+      qsort(col, (size_t)R, sizeof(int64_t), cmp_i64);
+      SPREAD[w * S + s] += col[R - 1] - col[(R - 1) / 2]; /* max minus lower median over ranks */
+    }
+  }
+  free(col);
+  return rc;
+}

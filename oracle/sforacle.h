@@ -94,6 +94,18 @@ int sfo_label_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t
 int sfo_baselines(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W, int64_t* M,
                   uint64_t* SUM, int64_t* SLOW, int64_t* RANK0);
 
+/* Localization evidence of Sec. 4, per step and stage: the lag
+     L[t,s] = F[t,s] - median_r P[t,r,s]   (lower median over ranks),
+   its increment dL[t,s] = L[t,s] - L[t,s-1] (L[t,-1] = 0), and the
+   max-minus-second-max gap G[t,s] = F[t,s] - (second largest P[t,r,s], a tie
+   at the top counting as the second; with R = 1 the gap is 0).
+   Outputs [T][S], each nullable. */
+int sfo_rank_lag(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t* L, int64_t* dL, int64_t* G);
+
+/* Raw rank spread of the Sec. 6 routing table, per window and stage:
+   sum_t (max_r d[t,r,s] - median_r d[t,r,s]), lower median over ranks. */
+int sfo_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W, int64_t* SPREAD);
+
 void sfo_config_default(sfo_config* cfg);
 
 #ifdef __cplusplus

@@ -200,6 +200,25 @@ sf_status sf_window_baselines(const int64_t* d, int64_t T, int64_t R, int64_t S,
   return cuda_status(launch_stream_pass(j, stream));
 }
 
+sf_status sf_rank_lag(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t* L, int64_t* dL, int64_t* G,
+                      uint32_t* status, cudaStream_t stream) {
+  if (!d || !shape_ok(T, R, S) || (!L && !dL && !G)) return SF_EINVAL;
+  if (!aligned(d, 16) || !aligned(L, 8) || !aligned(dL, 8) || !aligned(G, 8) || !aligned(status, 4))
+    return SF_EINVAL_ALIGN;
+  return cuda_status(launch_rank_select(d, T, R, S, 1, 0, 1, L, dL, G, nullptr, status, stream));
+}
+
+sf_status sf_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W, int64_t* spread,
+                        int32_t accumulate, uint32_t* status, cudaStream_t stream) {
+  if (!d || !spread || !shape_ok(T, R, S) || t0 < 0 || W < 1 || W > 65536 || (accumulate != 0 && accumulate != 1) ||
+      t0 > (int64_t(1) << 62) - T)
+    return SF_EINVAL;
+  if (!aligned(d, 16) || !aligned(spread, 8) || !aligned(status, 4)) return SF_EINVAL_ALIGN;
+  if (!accumulate && launch_zero(spread, size_t(sf_num_windows(t0, T, W)) * S * 8, stream) != cudaSuccess)
+    return SF_ECUDA;
+  return cuda_status(launch_rank_select(d, T, R, S, 0, t0, W, nullptr, nullptr, nullptr, spread, status, stream));
+}
+
 sf_status sf_topk_suspects(const int64_t* X, const int64_t* E, int64_t nW, int64_t S, int64_t R, int32_t k,
                            int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair,
                            int64_t* top_pair_value, cudaStream_t stream) {

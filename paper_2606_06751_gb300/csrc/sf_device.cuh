@@ -128,6 +128,45 @@ __device__ __forceinline__ uint64_t warp_min_u64(uint64_t v) {
   return (static_cast<uint64_t>(mhi) << 32) | mlo;
 }
 
+// Histogram scan of one radix pass: the digit d whose bin holds rank `rem`
+// among the counted values, and the count of values in lower bins.  Each lane
+// owns 8 consecutive bins; the lane whose range holds `rem` is found with one
+// warp scan and one ballot, and the bin within it by counting the inclusive
+// prefixes not above `rem` (every lane does the arithmetic; the owner's
+// result is broadcast).
+__device__ __forceinline__ void hist_find(const uint32_t* hist, uint32_t rem, int lane, uint32_t& digit,
+                                          uint32_t& below) {
+  const uint4 h0 = reinterpret_cast<const uint4*>(hist)[2 * lane];
+  const uint4 h1 = reinterpret_cast<const uint4*>(hist)[2 * lane + 1];
+  uint32_t c[8];  // inclusive prefix within the lane's 8 bins
+  c[0] = h0.x;
+  c[1] = c[0] + h0.y;
+  c[2] = c[1] + h0.z;
+  c[3] = c[2] + h0.w;
+  c[4] = c[3] + h1.x;
+  c[5] = c[4] + h1.y;
+  c[6] = c[5] + h1.z;
+  c[7] = c[6] + h1.w;
+  uint32_t incl = c[7];
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t up = __shfl_up_sync(kFull, incl, o);
+    if (lane >= o) incl += up;
+  }
+  const uint32_t excl = incl - c[7];
+  const int owner = __ffs(__ballot_sync(kFull, excl <= rem && rem < incl)) - 1;
+  const uint32_t r = rem - excl;  // rank within the owner's bins
+  uint32_t j = 0, bl = 0;
+#pragma unroll
+  for (int q = 0; q < 7; ++q) {
+    const bool past = c[q] <= r;  // bin q lies wholly below rank r
+    j += past ? 1u : 0u;
+    bl = past ? c[q] : bl;
+  }
+  digit = __shfl_sync(kFull, 8u * lane + j, owner);
+  below = __shfl_sync(kFull, excl + bl, owner);
+}
+
 __device__ __forceinline__ void report(uint32_t* status, uint32_t bits) {
   if (status != nullptr && bits != 0u) atomicOr(status, bits);
 }

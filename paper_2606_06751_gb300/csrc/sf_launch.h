@@ -57,6 +57,9 @@ cudaError_t launch_wait_selftest(uint64_t limit_ns, uint32_t* status, cudaStream
 cudaError_t launch_stream_pass(const StreamJob& job, cudaStream_t stream);
 cudaError_t launch_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W,
                                  int64_t* m, uint32_t* status, cudaStream_t stream);
+cudaError_t launch_rank_select(const int64_t* d, int64_t T, int64_t R, int64_t S, int of_prefix, int64_t t0,
+                               int64_t W, int64_t* L, int64_t* dL, int64_t* G, int64_t* spread, uint32_t* status,
+                               cudaStream_t stream);
 cudaError_t launch_topk(const int64_t* X, const int64_t* E, int64_t nW, int64_t S, int64_t R,
                         int32_t k, int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair,
                         int64_t* top_pair_value, cudaStream_t stream);

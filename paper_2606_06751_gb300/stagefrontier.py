@@ -54,6 +54,8 @@ def _load():
         "sf_window_aggregate": [P, I, I, I, I, I, P, P, P, P, P, I32, P, S],
         "sf_topk_suspects": [P, P, I, I, I, I32, P, P, P, P, S],
         "sf_window_baselines": [P, I, I, I, I, I, P, P, P, P, I32, P, S],
+        "sf_rank_lag": [P, I, I, I, P, P, P, P, S],
+        "sf_raw_spread": [P, I, I, I, I, I, P, I32, P, S],
         "sf_window_median": [P, I, I, I, I, P, P, S],
         "sf_direct_gain": [P, I, I, I, I, P, P, I32, Ratio, P, P, P, P, P, P, P, P, S],
         "sf_label_gates": [I, I, I, I, P, P, P, P, P, P, P, ctypes.POINTER(LabelConfig), P, P, P, P,
@@ -404,3 +406,27 @@ def sf_window_baselines(d, W: int, t0: int = 0, out: Optional[Baselines] = None,
     _check(_lib.sf_window_baselines(_p(d), T, R, S, t0, W, _p(out.M), _p(out.SUM), _p(out.SLOW), _p(out.RANK0),
                                     1 if accumulate else 0, _p(status), _stream(stream)), "sf_window_baselines")
     return out
+
+
+@dataclass
+class Lag:
+    L: Optional[torch.Tensor]   # [T][S] F - median_r P
+    dL: Optional[torch.Tensor]  # [T][S] increment of the lag over stages
+    G: Optional[torch.Tensor]   # [T][S] max-minus-second-max gap
+
+
+def sf_rank_lag(d, out: Optional[Lag] = None, status=None, stream=None) -> Lag:
+    T, R, S = _d3(d)
+    if out is None:
+        out = Lag(_empty((T, S), torch.int64, d), _empty((T, S), torch.int64, d), _empty((T, S), torch.int64, d))
+    _check(_lib.sf_rank_lag(_p(d), T, R, S, _p(out.L), _p(out.dL), _p(out.G), _p(status), _stream(stream)),
+           "sf_rank_lag")
+    return out
+
+
+def sf_raw_spread(d, W: int, t0: int = 0, spread=None, accumulate: bool = False, status=None, stream=None):
+    T, R, S = _d3(d)
+    spread = spread if spread is not None else _empty((num_windows(t0, T, W), S), torch.int64, d)
+    _check(_lib.sf_raw_spread(_p(d), T, R, S, t0, W, _p(spread), 1 if accumulate else 0, _p(status),
+                              _stream(stream)), "sf_raw_spread")
+    return spread

@@ -97,6 +97,13 @@ def test_host_validation(sf):
     assert dg(FAKE, 10, 4, 4, 5, FAKE, None, -1, sf.Ratio(1, 20), FAKE, FAKE, FAKE, FAKE + 4, None, FAKE,
               None, None, None) == sf.SF_EINVAL_ALIGN
     assert L.sf_window_median(FAKE, 10, 4, 4, 0, FAKE, None, None) == sf.SF_EINVAL
+    # cross-rank order statistics: no outputs, bad window, misaligned output
+    assert L.sf_rank_lag(FAKE, 10, 4, 4, None, None, None, None, None) == sf.SF_EINVAL
+    assert L.sf_rank_lag(FAKE, 10, 4, 4, FAKE + 4, None, None, None, None) == sf.SF_EINVAL_ALIGN
+    assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 0, FAKE, 0, None, None) == sf.SF_EINVAL
+    assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, None, 0, None, None) == sf.SF_EINVAL
+    assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, FAKE, 3, None, None) == sf.SF_EINVAL
+    assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, FAKE + 4, 0, None, None) == sf.SF_EINVAL_ALIGN
     # nothing was launched by any of the rejected calls
     assert sf.launch_count() == 0
 

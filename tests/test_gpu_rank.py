@@ -1,0 +1,132 @@
+"""GPU parity of the cross-rank order statistics: the Sec. 4 lag, its
+increment over stages and the max-minus-second-max gap per step, and the
+Sec. 6 raw rank spread per window, against the CPU oracle, bit-exact."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as O
+from synth import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def sf():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_06751_gb300 import build as B
+    B.build()
+    from paper_2606_06751_gb300 import stagefrontier
+    return stagefrontier
+
+
+def dev(x):
+    return torch.from_numpy(np.ascontiguousarray(x)).cuda()
+
+
+def host(t):
+    return t.cpu().numpy()
+
+
+def make(T, R, S, seed, kind):
+    rng = np.random.default_rng(seed)
+    if kind == "ties":
+        return rng.integers(0, 6, size=(T, R, S), dtype=np.int64)
+    if kind == "zeros":
+        d = rng.integers(0, 1000, size=(T, R, S), dtype=np.int64)
+        d[rng.random((T, R, S)) < 0.6] = 0
+        return d
+    if kind == "wide":      # offsets spanning 5-6 bytes: every radix pass runs
+        return rng.integers(0, 1 << 41, size=(T, R, S), dtype=np.int64)
+    med = rng.uniform(1e6, 5e7, size=S)
+    return np.rint(med * np.exp(0.1 * rng.standard_normal((T, R, S)))).astype(np.int64)
+
+
+# templated stage counts (4, 6, 8, 10, 16) and the generic kernel; R = 1 and 2,
+# odd and even R, R above the CTA width, the largest R
+SHAPES = [(20, 1, 1), (9, 2, 3), (37, 3, 5), (11, 7, 32), (6, 5, 18), (50, 2, 8),
+          (1000, 8, 6), (123, 64, 4), (97, 40, 10), (77, 64, 16), (31, 257, 8),
+          (13, 1024, 10), (7, 8192, 8), (5, 4096, 16), (3, 32768, 4), (2, 65536, 2), (2, 65535, 7)]
+
+
+@pytest.mark.parametrize("T,R,S", SHAPES)
+@pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal", "wide"])
+def test_rank_lag_parity(sf, T, R, S, kind):
+    d_np = make(T, R, S, T * 17 + R * 5 + S, kind)
+    o = O.rank_lag(d_np)
+    st = sf.new_status("cuda")
+    g = sf.sf_rank_lag(dev(d_np), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert np.array_equal(host(g.L), o.L)
+    assert np.array_equal(host(g.dL), o.dL)
+    assert np.array_equal(host(g.G), o.G)
+
+
+def test_rank_lag_optional_outputs(sf):
+    d_np = make(40, 33, 6, 5, "lognormal")
+    o = O.rank_lag(d_np)
+    d = dev(d_np)
+    only = sf.Lag(None, None, torch.empty((40, 6), dtype=torch.int64, device="cuda"))
+    sf.sf_rank_lag(d, out=only)
+    torch.cuda.synchronize()
+    assert np.array_equal(host(only.G), o.G)
+
+
+@pytest.mark.parametrize("T,R,S", [(20, 1, 1), (37, 3, 5), (301, 64, 4), (97, 40, 10), (1000, 8, 6),
+                                   (23, 1024, 10), (9, 8192, 8), (4, 65536, 2)])
+@pytest.mark.parametrize("t0,W", [(0, 1), (0, 7), (5, 10), (3, 1000)])
+def test_raw_spread_parity(sf, T, R, S, t0, W):
+    d_np = make(T, R, S, T + R + S + W, "ties" if R < 100 else "lognormal")
+    o = O.raw_spread(d_np, W, t0)
+    st = sf.new_status("cuda")
+    got = sf.sf_raw_spread(dev(d_np), W, t0=t0, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert np.array_equal(host(got), o)
+
+
+def test_raw_spread_accumulates_across_chunks(sf):
+    T, R, S, W = 2500, 128, 8, 1000
+    d_np = make(T, R, S, 11, "lognormal")
+    o = O.raw_spread(d_np, W)
+    out = torch.zeros((3, S), dtype=torch.int64, device="cuda")
+    for t0 in (0, 700, 1900):
+        t1 = {0: 700, 700: 1900, 1900: 2500}[t0]
+        w0 = t0 // W
+        part = out[w0:]
+        sf.sf_raw_spread(dev(d_np[t0:t1]), W, t0=t0, spread=part, accumulate=True)
+    torch.cuda.synchronize()
+    assert np.array_equal(host(out), o)
+
+
+def test_rank_lag_status_bits(sf):
+    d_np = make(8, 16, 4, 3, "lognormal")
+    d_np[3, 5, 2] = -1
+    st = sf.new_status("cuda")
+    sf.sf_rank_lag(dev(d_np), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & sf.SF_ST_NEGATIVE
+    d_np = make(8, 16, 4, 3, "lognormal")
+    d_np[2, 1, 1] = 1 << 50
+    st = sf.new_status("cuda")
+    sf.sf_raw_spread(dev(d_np), 4, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & sf.SF_ST_RANGE
+
+
+@pytest.mark.parametrize("name", ["tiny", "ddp128", "fsdp1024", "accum8192"])
+def test_rank_lag_on_workloads(sf, name):
+    """The workload generators (sync stages absorbing skew, stalls, Pareto
+    tails, node slowdowns) on a prefix of steps, lag and spread exact."""
+    w = wl.by_name(name)
+    n = {"tiny": 1000, "ddp128": 3000, "fsdp1024": 600, "accum8192": 40}[name]
+    d_np = w.generate(0, n)
+    o = O.rank_lag(d_np)
+    g = sf.sf_rank_lag(dev(d_np))
+    sp = sf.sf_raw_spread(dev(d_np), w.W)
+    torch.cuda.synchronize()
+    assert np.array_equal(host(g.L), o.L) and np.array_equal(host(g.dL), o.dL)
+    assert np.array_equal(host(g.G), o.G)
+    assert np.array_equal(host(sp), O.raw_spread(d_np, w.W))

@@ -460,3 +460,49 @@ def test_baselines_big_sums_are_exact():
     d = np.full((4, 3, 1), (1 << 46) + 12345, np.int64)  # each rank total just under 2^47
     b = O.baselines(d, 4)
     assert b.SUM[0][0] == 12 * ((1 << 46) + 12345)    # above 2^49, exact
+
+
+# ---------------------------------------------------------------- localization evidence (Sec. 4) and spread (Sec. 6)
+
+@pytest.mark.parametrize("seed", range(3))
+def test_lag_against_library_routines(seed):
+    rng = np.random.default_rng(600 + seed)
+    T, R, S = 20, 9, 5                                   # odd R: lower median == np.median
+    d = rand_d(rng, T, R, S, hi=50, zero_frac=0.2)
+    g = O.rank_lag(d)
+    P = np.cumsum(d, axis=2)
+    F = P.max(axis=1)
+    assert (g.L == F - np.median(P, axis=1).astype(np.int64)).all()
+    assert (g.G == F - np.sort(P, axis=1)[:, -2, :]).all()
+    assert (g.dL == np.diff(np.concatenate([np.zeros((T, 1), np.int64), g.L], axis=1), axis=1)).all()
+    assert (g.L >= 0).all() and (g.G >= 0).all()
+    assert (F == O.frontier(d).F).all()                  # the lag's maximum is the frontier
+
+
+def test_lag_special_cases():
+    rng = np.random.default_rng(3)
+    one = rand_d(rng, 6, 1, 4)
+    g = O.rank_lag(one)
+    assert (g.L == 0).all() and (g.G == 0).all()          # R = 1: no cross-rank evidence
+    same = np.repeat(rand_d(rng, 6, 1, 4), 5, axis=1)
+    g = O.rank_lag(same)
+    assert (g.L == 0).all() and (g.G == 0).all()          # identical ranks: no lag, tied top
+    # a stall Delta on one rank of otherwise identical ranks (R >= 3, no sync):
+    # from the stalled stage on, the lag and the gap are both exactly Delta
+    base = rng.integers(1, 1000, size=4).astype(np.int64)
+    d = np.tile(base, (1, 5, 1))
+    d[0, 2, 1] += 777
+    g = O.rank_lag(d)
+    assert list(g.L[0]) == [0, 777, 777, 777] and list(g.G[0]) == [0, 777, 777, 777]
+    assert list(g.dL[0]) == [0, 777, 0, 0]
+
+
+def test_raw_spread():
+    rng = np.random.default_rng(11)
+    T, R, S, W = 30, 7, 4, 8
+    d = rand_d(rng, T, R, S, hi=100)
+    sp = O.raw_spread(d, W)
+    per_step = d.max(axis=1) - np.median(d, axis=1).astype(np.int64)
+    for w in range(sp.shape[0]):
+        assert (sp[w] == per_step[w * W:(w + 1) * W].sum(axis=0)).all()
+    assert (O.raw_spread(np.repeat(d[:, :1], 5, axis=1), W) == 0).all()
