@@ -130,23 +130,16 @@ __device__ __forceinline__ uint64_t warp_min_u64(uint64_t v) {
 
 // Histogram scan of one radix pass: the digit d whose bin holds rank `rem`
 // among the counted values, and the count of values in lower bins.  Each lane
-// owns 8 consecutive bins; the lane whose range holds `rem` is found with one
-// warp scan and one ballot, and the bin within it by counting the inclusive
-// prefixes not above `rem` (every lane does the arithmetic; the owner's
-// result is broadcast).
-__device__ __forceinline__ void hist_find(const uint32_t* hist, uint32_t rem, int lane, uint32_t& digit,
+// owns 8 consecutive bins (h[0..7] = bins 8*lane .. 8*lane+7); the lane whose
+// range holds `rem` is found with one warp scan and one ballot, and the bin
+// within it by counting the inclusive prefixes not above `rem` (every lane
+// does the arithmetic; the owner's result is broadcast).
+__device__ __forceinline__ void bins_find(const uint32_t (&h)[8], uint32_t rem, int lane, uint32_t& digit,
                                           uint32_t& below) {
-  const uint4 h0 = reinterpret_cast<const uint4*>(hist)[2 * lane];
-  const uint4 h1 = reinterpret_cast<const uint4*>(hist)[2 * lane + 1];
   uint32_t c[8];  // inclusive prefix within the lane's 8 bins
-  c[0] = h0.x;
-  c[1] = c[0] + h0.y;
-  c[2] = c[1] + h0.z;
-  c[3] = c[2] + h0.w;
-  c[4] = c[3] + h1.x;
-  c[5] = c[4] + h1.y;
-  c[6] = c[5] + h1.z;
-  c[7] = c[6] + h1.w;
+  c[0] = h[0];
+#pragma unroll
+  for (int q = 1; q < 8; ++q) c[q] = c[q - 1] + h[q];
   uint32_t incl = c[7];
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
@@ -165,6 +158,15 @@ __device__ __forceinline__ void hist_find(const uint32_t* hist, uint32_t rem, in
   }
   digit = __shfl_sync(kFull, 8u * lane + j, owner);
   below = __shfl_sync(kFull, excl + bl, owner);
+}
+
+// bins_find over a 256-bin shared-memory histogram (16-byte aligned).
+__device__ __forceinline__ void hist_find(const uint32_t* hist, uint32_t rem, int lane, uint32_t& digit,
+                                          uint32_t& below) {
+  const uint4 h0 = reinterpret_cast<const uint4*>(hist)[2 * lane];
+  const uint4 h1 = reinterpret_cast<const uint4*>(hist)[2 * lane + 1];
+  const uint32_t h[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+  bins_find(h, rem, lane, digit, below);
 }
 
 __device__ __forceinline__ void report(uint32_t* status, uint32_t bits) {

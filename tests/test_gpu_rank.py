@@ -40,18 +40,23 @@ def make(T, R, S, seed, kind):
     if kind == "wide":      # offsets spanning 5-6 bytes: every radix pass runs
         return rng.integers(0, 1 << 41, size=(T, R, S), dtype=np.int64)
     med = rng.uniform(1e6, 5e7, size=S)
-    return np.rint(med * np.exp(0.1 * rng.standard_normal((T, R, S)))).astype(np.int64)
+    d = np.rint(med * np.exp(0.1 * rng.standard_normal((T, R, S)))).astype(np.int64)
+    if kind == "mixed":     # a few steps with a multi-second stall on one rank (64-bit path)
+        for t in rng.choice(T, size=max(1, T // 7), replace=False):
+            d[t, rng.integers(R), rng.integers(S)] += int(rng.integers(1 << 31, 1 << 33))
+    return d
 
 
 # templated stage counts (4, 6, 8, 10, 16) and the generic kernel; R = 1 and 2,
 # odd and even R, R above the CTA width, the largest R
 SHAPES = [(20, 1, 1), (9, 2, 3), (37, 3, 5), (11, 7, 32), (6, 5, 18), (50, 2, 8),
           (1000, 8, 6), (123, 64, 4), (97, 40, 10), (77, 64, 16), (31, 257, 8),
-          (13, 1024, 10), (7, 8192, 8), (5, 4096, 16), (3, 32768, 4), (2, 65536, 2), (2, 65535, 7)]
+          (13, 1024, 10), (7, 8192, 8), (5, 4096, 16), (3, 32768, 4), (2, 65536, 2), (2, 65535, 7),
+          (2, 32768, 16), (3, 9000, 9)]
 
 
 @pytest.mark.parametrize("T,R,S", SHAPES)
-@pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal", "wide"])
+@pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal", "wide", "mixed"])
 def test_rank_lag_parity(sf, T, R, S, kind):
     d_np = make(T, R, S, T * 17 + R * 5 + S, kind)
     o = O.rank_lag(d_np)
