@@ -82,6 +82,10 @@ def lib():
         L.sfo_rank_lag.restype = ctypes.c_int
         L.sfo_raw_spread.argtypes = [_P, _I, _I, _I, _I, _I, _P]
         L.sfo_raw_spread.restype = ctypes.c_int
+        L.sfo_group_windows.argtypes = [_P, _I, _I, _I, _P, _I, _I, _I, _P, _P]
+        L.sfo_group_windows.restype = ctypes.c_int
+        L.sfo_stage_group_sum.argtypes = [_P, _I, _I, _P, _I, _P]
+        L.sfo_stage_group_sum.restype = ctypes.c_int
         L.sfo_config_default.argtypes = [ctypes.POINTER(Config)]
         for f in ("sfo_frontier", "sfo_windows", "sfo_topk", "sfo_window_median", "sfo_direct_gain",
                   "sfo_label_windows"):
@@ -283,3 +287,32 @@ def raw_spread(d, W: int, t0: int = 0) -> np.ndarray:
     out = np.empty((num_windows(t0, T, W), S), np.int64)
     _check(lib().sfo_raw_spread(_ptr(d), T, R, S, t0, W, _ptr(out)))
     return out
+
+
+@dataclass
+class GroupWindows:
+    X: np.ndarray  # [G][nW][S] sum of the group frontier's increments
+    D: np.ndarray  # [G][nW] sum of the group makespans
+
+
+def group_windows(d, group, G: int, W: int, t0: int = 0) -> GroupWindows:
+    """Frontier within role groups (App. A role check, Sec. 3 Eq. 1 per group)."""
+    d = _d(d)
+    T, R, S = d.shape
+    group = np.ascontiguousarray(group, dtype=np.int32)
+    assert group.shape == (R,)
+    nW = num_windows(t0, T, W)
+    out = GroupWindows(np.empty((G, nW, S), np.int64), np.empty((G, nW), np.int64))
+    _check(lib().sfo_group_windows(_ptr(d), T, R, S, _ptr(group), G, t0, W, _ptr(out.X), _ptr(out.D)))
+    return out
+
+
+def stage_group_sum(X, stage_group, K: int) -> np.ndarray:
+    """Reporting groups aggregated after the frontier (Sec. 3)."""
+    X = np.ascontiguousarray(X, dtype=np.int64)
+    nW, S = X.shape
+    stage_group = np.ascontiguousarray(stage_group, dtype=np.int32)
+    assert stage_group.shape == (S,)
+    Y = np.empty((nW, K), np.int64)
+    _check(lib().sfo_stage_group_sum(_ptr(X), nW, S, _ptr(stage_group), K, _ptr(Y)))
+    return Y

@@ -494,3 +494,58 @@ int sfo_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0
   free(col);
   return rc;
 }
+
+int sfo_group_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, const int32_t* group, int64_t G,
+                      int64_t t0, int64_t W, int64_t* Xg, int64_t* Dg) {
+  if (!d || !group || !check_shape(T, R, S) || G < 1 || G > 65536 || W < 1 || W > 65536 || t0 < 0 || !Xg ||
+      !Dg)
+    return SFO_BADARG;
+  for (int64_t r = 0; r < R; ++r)
+    if (group[r] < 0 || group[r] >= G) return SFO_BADARG;
+  int64_t w_first = floordiv(t0, W);
+  int64_t nW = floordiv(t0 + T - 1, W) - w_first + 1;
+  memset(Xg, 0, sizeof(int64_t) * (size_t)(G * nW * S));
+  memset(Dg, 0, sizeof(int64_t) * (size_t)(G * nW));
+  int64_t* P = (int64_t*)malloc(sizeof(int64_t) * (size_t)R);
+  int64_t* Fg = (int64_t*)malloc(sizeof(int64_t) * (size_t)G);     /* F_g[t,s] at the current s */
+  int64_t* Fprev = (int64_t*)malloc(sizeof(int64_t) * (size_t)G);  /* F_g[t,s-1] */
+  int rc = (P && Fg && Fprev) ? SFO_OK : SFO_BADARG;
+  for (int64_t t = 0; t < T && rc == SFO_OK; ++t) {
+    const int64_t* dt = d + t * R * S;
+    int64_t w = floordiv(t0 + t, W) - w_first;
+    for (int64_t r = 0; r < R; ++r) P[r] = 0;
+    for (int64_t g = 0; g < G; ++g) Fprev[g] = 0;
+    for (int64_t s = 0; s < S && rc == SFO_OK; ++s) {
+      for (int64_t g = 0; g < G; ++g) Fg[g] = 0;
+      for (int64_t r = 0; r < R; ++r) {
+        int64_t v = dt[r * S + s];
+        if (v < 0) { rc = SFO_NEGATIVE; break; }
+        if (v >= LIMIT47) { rc = SFO_RANGE; break; }
+        P[r] += v;
+        if (P[r] > Fg[group[r]]) Fg[group[r]] = P[r]; /* max over the group's ranks */
+      }
+      for (int64_t g = 0; g < G && rc == SFO_OK; ++g) {
+        Xg[(g * nW + w) * S + s] += Fg[g] - Fprev[g]; /* a_g[t,s] */
+        Fprev[g] = Fg[g];
+      }
+    }
+    for (int64_t r = 0; r < R && rc == SFO_OK; ++r)
+      if (P[r] >= LIMIT47) rc = SFO_RANGE;
+    for (int64_t g = 0; g < G && rc == SFO_OK; ++g) Dg[g * nW + w] += Fprev[g]; /* F_g[t,S-1] */
+  }
+  free(P);
+  free(Fg);
+  free(Fprev);
+  return rc;
+}
+
+int sfo_stage_group_sum(const int64_t* X, int64_t nW, int64_t S, const int32_t* stage_group, int64_t K,
+                        int64_t* Y) {
+  if (!X || !stage_group || !Y || nW < 0 || S < 1 || S > 32 || K < 1 || K > 32) return SFO_BADARG;
+  for (int64_t s = 0; s < S; ++s)
+    if (stage_group[s] < 0 || stage_group[s] >= K) return SFO_BADARG;
+  memset(Y, 0, sizeof(int64_t) * (size_t)(nW * K));
+  for (int64_t w = 0; w < nW; ++w)
+    for (int64_t s = 0; s < S; ++s) Y[w * K + stage_group[s]] += X[w * S + s];
+  return SFO_OK;
+}

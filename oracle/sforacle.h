@@ -108,6 +108,22 @@ int sfo_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0
 
 void sfo_config_default(sfo_config* cfg);
 
+/* Frontier within role groups (App. A role check: no global frontier across
+   incompatible roles; Sec. 3 Eq. 1 applied inside each group).  group [R]
+   gives each rank's group in [0, G).  For every group g and step t:
+     F_g[t,s] = max of P[t,r,s] over the ranks r of g (0 for a group with no rank),
+     a_g[t,s] = F_g[t,s] - F_g[t,s-1] with F_g[t,-1] = 0.
+   Per window (t0, W as in sfo_windows): Xg [G][nW][S] = sum of a_g over the
+   window's steps, Dg [G][nW] = sum of F_g[t,S-1].  Outputs overwritten. */
+int sfo_group_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, const int32_t* group, int64_t G,
+                      int64_t t0, int64_t W, int64_t* Xg, int64_t* Dg);
+
+/* Reporting groups aggregated after the frontier (Sec. 3, accumulation
+   expansion): Y [nW][K] = sum of X[w][s] over the stages s with
+   stage_group[s] = k, stage_group [S] in [0, K). */
+int sfo_stage_group_sum(const int64_t* X, int64_t nW, int64_t S, const int32_t* stage_group, int64_t K,
+                        int64_t* Y);
+
 #ifdef __cplusplus
 }
 #endif

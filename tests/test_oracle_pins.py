@@ -506,3 +506,57 @@ def test_raw_spread():
     for w in range(sp.shape[0]):
         assert (sp[w] == per_step[w * W:(w + 1) * W].sum(axis=0)).all()
     assert (O.raw_spread(np.repeat(d[:, :1], 5, axis=1), W) == 0).all()
+
+
+# ---------------------------------------------------------------- role groups (App. A) and reporting groups (Sec. 3)
+
+@pytest.mark.parametrize("seed", range(3))
+def test_group_windows_one_group_is_the_global_frontier(seed):
+    rng = np.random.default_rng(700 + seed)
+    T, R, S, W = 25, 6, 4, 7
+    d = rand_d(rng, T, R, S, hi=80, zero_frac=0.2)
+    gw = O.group_windows(d, np.zeros(R, np.int32), 1, W, t0=3)
+    w = O.windows(d, W, t0=3)
+    assert (gw.X[0] == w.X).all() and (gw.D[0] == w.D).all()
+
+
+def test_group_windows_singletons_are_rank_sums():
+    # one rank per group: the group frontier is the rank's own prefix, so the
+    # increments are its durations and the makespan its total
+    rng = np.random.default_rng(5)
+    T, R, S, W = 12, 5, 3, 4
+    d = rand_d(rng, T, R, S, hi=60)
+    gw = O.group_windows(d, np.arange(R, dtype=np.int32), R, W)
+    for g in range(R):
+        for w in range(gw.X.shape[1]):
+            assert (gw.X[g, w] == d[w * W:(w + 1) * W, g, :].sum(axis=0)).all()
+            assert gw.D[g, w] == d[w * W:(w + 1) * W, g, :].sum()
+
+
+def test_group_windows_invariants_and_empty_groups():
+    rng = np.random.default_rng(9)
+    T, R, S, W = 40, 9, 5, 10
+    d = rand_d(rng, T, R, S, hi=50, zero_frac=0.3)
+    group = rng.integers(0, 3, size=R).astype(np.int32)
+    group[group == 2] = 1                                # group 2 left empty, group 3 too
+    gw = O.group_windows(d, group, 4, W)
+    w = O.windows(d, W)
+    assert (gw.X >= 0).all()                             # group frontiers are monotone in s
+    assert (gw.X.sum(axis=2) == gw.D).all()              # Theorem 1 inside each group
+    assert (gw.X[2] == 0).all() and (gw.D[2] == 0).all() and (gw.D[3] == 0).all()
+    assert (gw.D <= w.D).all() and (w.D <= gw.D.sum(axis=0)).all()
+    # permuting ranks together with their group ids changes nothing
+    perm = rng.permutation(R)
+    gp = O.group_windows(d[:, perm, :], group[perm], 4, W)
+    assert (gp.X == gw.X).all() and (gp.D == gw.D).all()
+
+
+def test_stage_group_sum():
+    rng = np.random.default_rng(4)
+    d = rand_d(rng, 30, 4, 8, hi=90)
+    w = O.windows(d, 10)
+    assert (O.stage_group_sum(w.X, np.arange(8), 8) == w.X).all()          # singletons: identity
+    assert (O.stage_group_sum(w.X, np.zeros(8), 1)[:, 0] == w.D).all()     # one group: Theorem 1
+    fb = np.array([0, 1] * 4)                                              # f1 b1 f2 b2 ... -> fwd, bwd
+    y = O.stage_group_sum(w.X, fb, 2)
+    assert (y[:, 0] == w.X[:, 0::2].sum(axis=1)).all() and (y.sum(axis=1) == w.D).all()
