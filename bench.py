@@ -231,6 +231,10 @@ class Pipeline:
                                  e((nW, S), torch.int64))
         self.lag = sf.Lag(e((T, S), torch.int64), e((T, S), torch.int64), e((T, S), torch.int64))
         self.spread = e((nW, S), torch.int64)
+        # role groups: nodes of 128 consecutive ranks (one group when R <= 128)
+        self.n_groups = max(1, R // 128)
+        self.node_group = (torch.arange(R, device=dev, dtype=torch.int32) * self.n_groups // R).to(torch.int32)
+        self.grp = sf.GroupWindows(e((nW, self.n_groups, S), torch.int64), e((nW, self.n_groups), torch.int64))
         self.status = sf.new_status(dev)
         self.names = ["window_median", "direct_gain", "topk_suspects", "label_gates"]
         self.events = None
@@ -273,6 +277,11 @@ class Pipeline:
         """The raw rank spread per window (sf_raw_spread)."""
         self.sf.sf_raw_spread(self.d, self.w.W, spread=self.spread, status=self.status)
 
+    def group_aggregate(self):
+        """The frontier within node groups of 128 ranks (sf_group_aggregate)."""
+        self.sf.sf_group_aggregate(self.d, self.node_group, self.n_groups, self.w.W, out=self.grp,
+                                   status=self.status)
+
     def results(self):
         return [self.lab.labels, self.lab.route_mask, self.lab.amb_mask, self.lab.share, self.lab.gain,
                 self.top.stage, self.top.pair, self.top.pair_value, self.ev.X, self.ev.D]
@@ -289,6 +298,7 @@ class Pipeline:
             "window_baselines": din + nW * w.S * 40 + w.T * w.S * 16,
             "rank_lag": din + 3 * w.T * w.S * 8,
             "raw_spread": din + nW * w.S * 8,
+            "group_aggregate": din + w.R * 4 + nW * self.n_groups * (w.S + 1) * 8,
         }
 
 
@@ -339,6 +349,7 @@ def run_ours(args):
     base_secs = timed_loop(pipe.baselines, args.steps, args.warmup, ws, device, True) / args.steps
     lag_secs = timed_loop(pipe.rank_lag, args.steps, args.warmup, ws, device, True) / args.steps
     spread_secs = timed_loop(pipe.raw_spread, args.steps, args.warmup, ws, device, True) / args.steps
+    group_secs = timed_loop(pipe.group_aggregate, args.steps, args.warmup, ws, device, True) / args.steps
 
     # end to end through the host-memory entry point: every step streams the
     # pinned host tensor to the GPU in 2000-step chunks (copies overlapping the
@@ -396,6 +407,9 @@ def run_ours(args):
         "spread_pass": {"entry": "sf_raw_spread", "ms": round(spread_secs * 1e3, 4),
                         "gbs": round(algo["raw_spread"] / spread_secs / 1e9, 1),
                         "frac": round(algo["raw_spread"] / spread_secs / 1e9 / peak, 4)},
+        "group_pass": {"entry": "sf_group_aggregate", "groups": pipe.n_groups, "ms": round(group_secs * 1e3, 4),
+                       "gbs": round(algo["group_aggregate"] / group_secs / 1e9, 1),
+                       "frac": round(algo["group_aggregate"] / group_secs / 1e9 / peak, 4)},
         "gpu_launches": int(launches * args.steps // (args.steps + args.warmup)),
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": w.nbytes, "d2h_bytes_per_step": d2h,
                 "entry": "sf_stream_windows", "chunk_steps": chunk},

@@ -57,6 +57,7 @@ typedef enum sf_status {
 #define SF_ST_NEGATIVE 1u /* some duration (or wall time) was negative */
 #define SF_ST_RANGE 2u    /* some duration, rank total or wall time was >= 2^47 */
 #define SF_ST_TIMEOUT 4u  /* a bounded device-side wait gave up; outputs incomplete */
+#define SF_ST_INDEX 8u    /* an index input (a rank's group id) was out of range; that rank was skipped */
 
 /* Label bits (Sec. 4 Tab. core labels, App. B, App. C).  RAW_ONLY marks a
    window whose denominator is below the floor: raw advances, no shares. */
@@ -155,6 +156,35 @@ sf_status sf_rank_lag(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t
  */
 sf_status sf_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W,
                         int64_t* spread, int32_t accumulate, uint32_t* status, cudaStream_t stream);
+
+/*
+ * sf_group_aggregate - the frontier taken within role groups.  The App. A
+ * contract check forbids one global frontier across ranks whose roles
+ * differ (the labeler then emits role_aware_needed); with a rank -> group
+ * map the frontier of Sec. 3 Eq. 1 is taken inside each group instead:
+ *   F_g[t,s] = max of P[t,r,s] over the ranks r of group g (0 if g has none),
+ *   a_g[t,s] = F_g[t,s] - F_g[t,s-1], F_g[t,-1] = 0,
+ *   Xg [nW][G][S] sum_t a_g[t,s],  Dg [nW][G] sum_t F_g[t,S-1]   (device, required)
+ * group [R] int32 device: each rank's group in [0, G); a rank whose id is
+ * outside that range is left out and SF_ST_INDEX is set.  1 <= G <= 4096,
+ * G*S <= 4096.  Windows, t0 and accumulate as in sf_window_aggregate.  The
+ * group Xg[:, g, :], Dg[:, g] feed sf_label_gates like X, D.
+ */
+sf_status sf_group_aggregate(const int64_t* d, int64_t T, int64_t R, int64_t S, const int32_t* group, int64_t G,
+                             int64_t t0, int64_t W, int64_t* Xg, int64_t* Dg, int32_t accumulate, uint32_t* status,
+                             cudaStream_t stream);
+
+/*
+ * sf_stage_group_sum - reporting groups aggregated after the frontier
+ * (Sec. 3: with gradient accumulation the ordered stage list is expanded by
+ * accumulation index before the frontier, and semantic groups such as
+ * "forward" or "backward" are summed only afterwards):
+ *   Y [nW][K] = sum of X[w][s] over the stages s with stage_group[s] = k.
+ * X [nW][S] device; stage_group [S] HOST array, values in [0, K), 1 <= K <= 32;
+ * Y device, overwritten.  nW = 0 is a no-op.
+ */
+sf_status sf_stage_group_sum(const int64_t* X, int64_t nW, int64_t S, const int32_t* stage_group, int64_t K,
+                             int64_t* Y, cudaStream_t stream);
 
 /*
  * sf_topk_suspects - per window, the k stages with the largest X (Sec. 4

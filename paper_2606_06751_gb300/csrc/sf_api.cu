@@ -219,6 +219,32 @@ sf_status sf_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64
   return cuda_status(launch_rank_select(d, T, R, S, 0, t0, W, nullptr, nullptr, nullptr, spread, status, stream));
 }
 
+sf_status sf_group_aggregate(const int64_t* d, int64_t T, int64_t R, int64_t S, const int32_t* group, int64_t G,
+                             int64_t t0, int64_t W, int64_t* Xg, int64_t* Dg, int32_t accumulate, uint32_t* status,
+                             cudaStream_t stream) {
+  if (!d || !group || !Xg || !Dg || !shape_ok(T, R, S) || G < 1 || G > 4096 || G * S > 4096 || t0 < 0 || W < 1 ||
+      W > 65536 || (accumulate != 0 && accumulate != 1) || t0 > (int64_t(1) << 62) - T)
+    return SF_EINVAL;
+  if (!aligned(d, 16) || !aligned(group, 4) || !aligned(Xg, 8) || !aligned(Dg, 8) || !aligned(status, 4))
+    return SF_EINVAL_ALIGN;
+  const size_t nW = size_t(sf_num_windows(t0, T, W));
+  if (!accumulate && (launch_zero(Xg, nW * G * S * 8, stream) != cudaSuccess ||
+                      launch_zero(Dg, nW * G * 8, stream) != cudaSuccess))
+    return SF_ECUDA;
+  return cuda_status(launch_group_windows(d, T, R, S, group, G, t0, W, Xg, Dg, status, stream));
+}
+
+sf_status sf_stage_group_sum(const int64_t* X, int64_t nW, int64_t S, const int32_t* stage_group, int64_t K,
+                             int64_t* Y, cudaStream_t stream) {
+  if (!X || !stage_group || !Y || nW < 0 || S < 1 || S > 32 || K < 1 || K > 32 || nW > (int64_t(1) << 40))
+    return SF_EINVAL;
+  for (int64_t s = 0; s < S; ++s)
+    if (stage_group[s] < 0 || stage_group[s] >= K) return SF_EINVAL;
+  if (!aligned(X, 8) || !aligned(Y, 8)) return SF_EINVAL_ALIGN;
+  if (nW == 0) return SF_OK;
+  return cuda_status(launch_stage_group_sum(X, nW, S, stage_group, K, Y, stream));
+}
+
 sf_status sf_topk_suspects(const int64_t* X, const int64_t* E, int64_t nW, int64_t S, int64_t R, int32_t k,
                            int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair,
                            int64_t* top_pair_value, cudaStream_t stream) {

@@ -60,6 +60,11 @@ cudaError_t launch_window_median(const int64_t* d, int64_t T, int64_t R, int64_t
 cudaError_t launch_rank_select(const int64_t* d, int64_t T, int64_t R, int64_t S, int of_prefix, int64_t t0,
                                int64_t W, int64_t* L, int64_t* dL, int64_t* G, int64_t* spread, uint32_t* status,
                                cudaStream_t stream);
+cudaError_t launch_group_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, const int32_t* group, int64_t G,
+                                 int64_t t0, int64_t W, int64_t* Xg, int64_t* Dg, uint32_t* status,
+                                 cudaStream_t stream);
+cudaError_t launch_stage_group_sum(const int64_t* X, int64_t nW, int64_t S, const int32_t* stage_group, int64_t K,
+                                   int64_t* Y, cudaStream_t stream);
 cudaError_t launch_topk(const int64_t* X, const int64_t* E, int64_t nW, int64_t S, int64_t R,
                         int32_t k, int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair,
                         int64_t* top_pair_value, cudaStream_t stream);

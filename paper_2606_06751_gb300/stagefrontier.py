@@ -20,7 +20,7 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libstagefrontier.so")
 
 SF_OK, SF_EINVAL, SF_EINVAL_ALIGN, SF_EUNSUPPORTED, SF_ECUDA, SF_EWORKSPACE = 0, -1, -2, -3, -4, -5
-SF_ST_NEGATIVE, SF_ST_RANGE, SF_ST_TIMEOUT = 1, 2, 4
+SF_ST_NEGATIVE, SF_ST_RANGE, SF_ST_TIMEOUT, SF_ST_INDEX = 1, 2, 4, 8
 SF_STEP_CONFIDENT = 0x80
 LABEL_NAMES = ("frontier_accounting", "direct_exposure", "sync_wait_dependent", "co_critical",
                "role_aware_needed", "telemetry_limited", "raw_only")
@@ -55,6 +55,8 @@ def _load():
         "sf_topk_suspects": [P, P, I, I, I, I32, P, P, P, P, S],
         "sf_window_baselines": [P, I, I, I, I, I, P, P, P, P, I32, P, S],
         "sf_rank_lag": [P, I, I, I, P, P, P, P, S],
+        "sf_group_aggregate": [P, I, I, I, P, I, I, I, P, P, I32, P, S],
+        "sf_stage_group_sum": [P, I, I, P, I, P, S],
         "sf_raw_spread": [P, I, I, I, I, I, P, I32, P, S],
         "sf_window_median": [P, I, I, I, I, P, P, S],
         "sf_direct_gain": [P, I, I, I, I, P, P, I32, Ratio, P, P, P, P, P, P, P, P, S],
@@ -430,3 +432,30 @@ def sf_raw_spread(d, W: int, t0: int = 0, spread=None, accumulate: bool = False,
     _check(_lib.sf_raw_spread(_p(d), T, R, S, t0, W, _p(spread), 1 if accumulate else 0, _p(status),
                               _stream(stream)), "sf_raw_spread")
     return spread
+
+
+@dataclass
+class GroupWindows:
+    X: torch.Tensor  # [nW][G][S] sums of the group frontier's increments
+    D: torch.Tensor  # [nW][G] sums of the group makespans
+
+
+def sf_group_aggregate(d, group, G: int, W: int, t0: int = 0, out: Optional[GroupWindows] = None,
+                       accumulate: bool = False, status=None, stream=None) -> GroupWindows:
+    T, R, S = _d3(d)
+    group = _dev(group, torch.int32, "group")
+    nW = num_windows(t0, T, W)
+    if out is None:
+        out = GroupWindows(_empty((nW, G, S), torch.int64, d), _empty((nW, G), torch.int64, d))
+    _check(_lib.sf_group_aggregate(_p(d), T, R, S, _p(group), G, t0, W, _p(out.X), _p(out.D),
+                                   1 if accumulate else 0, _p(status), _stream(stream)), "sf_group_aggregate")
+    return out
+
+
+def sf_stage_group_sum(X, stage_group, K: int, Y=None, stream=None):
+    """stage_group: a host sequence of S group ids in [0, K)."""
+    nW, S = X.shape
+    sg = (ctypes.c_int32 * S)(*[int(v) for v in stage_group])
+    Y = Y if Y is not None else _empty((nW, K), torch.int64, X)
+    _check(_lib.sf_stage_group_sum(_p(X), nW, S, sg, K, _p(Y), _stream(stream)), "sf_stage_group_sum")
+    return Y

@@ -104,6 +104,17 @@ def test_host_validation(sf):
     assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, None, 0, None, None) == sf.SF_EINVAL
     assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, FAKE, 3, None, None) == sf.SF_EINVAL
     assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, FAKE + 4, 0, None, None) == sf.SF_EINVAL_ALIGN
+    # role groups: group count, G*S limit, stage-group ids (host array)
+    ga = L.sf_group_aggregate
+    assert ga(FAKE, 10, 4, 4, FAKE, 0, 0, 5, FAKE, FAKE, 0, None, None) == sf.SF_EINVAL
+    assert ga(FAKE, 10, 4, 8, FAKE, 1000, 0, 5, FAKE, FAKE, 0, None, None) == sf.SF_EINVAL
+    assert ga(FAKE, 10, 4, 4, None, 2, 0, 5, FAKE, FAKE, 0, None, None) == sf.SF_EINVAL
+    assert ga(FAKE, 10, 4, 4, FAKE + 2, 2, 0, 5, FAKE, FAKE, 0, None, None) == sf.SF_EINVAL_ALIGN
+    sg = (ctypes.c_int32 * 4)(0, 1, 0, 5)
+    assert L.sf_stage_group_sum(FAKE, 3, 4, sg, 2, FAKE, None) == sf.SF_EINVAL
+    sg = (ctypes.c_int32 * 4)(0, 1, 0, 1)
+    assert L.sf_stage_group_sum(FAKE, 3, 4, sg, 33, FAKE, None) == sf.SF_EINVAL
+    assert L.sf_stage_group_sum(FAKE + 4, 3, 4, sg, 2, FAKE, None) == sf.SF_EINVAL_ALIGN
     # nothing was launched by any of the rejected calls
     assert sf.launch_count() == 0
 
