@@ -32,6 +32,7 @@ import re
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -115,7 +116,8 @@ class ClockSampler:
     def __init__(self, gpu_id: str):
         self.gpu = gpu_id
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_gpu{os.getpid()}.csv")
+        # raw samples go to SF_CLOCKS_DIR (default: the system temp directory)
+        self.path = os.path.join(os.environ.get("SF_CLOCKS_DIR", tempfile.gettempdir()), f"clocks_gpu{os.getpid()}.csv")
 
     def __enter__(self):
         try:

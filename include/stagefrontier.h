@@ -303,7 +303,7 @@ sf_status sf_label_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, in
  * E/C are given), sf_topk_suspects and sf_label_gates, its windows written to
  * the output rows they belong to.  The copy of the next chunk overlaps the
  * computation of the current one when h_d is page-locked and the two streams
- * differ.  This is the SURVEY's chunked streaming of the largest workload
+ * differ.  This is the chunked streaming of the largest workload
  * (Sec. 5's window-boundary delivery of rank vectors, here host to GPU).
  *   h_d        [T][R][S] host, 16-byte aligned (page-locked for overlap).
  *   staging    device, >= sf_stream_windows_staging_size(T, R, S, chunk_steps)
