@@ -353,6 +353,22 @@ def run_ours(args):
     spread_secs = timed_loop(pipe.raw_spread, args.steps, args.warmup, ws, device, True) / args.steps
     group_secs = timed_loop(pipe.group_aggregate, args.steps, args.warmup, ws, device, True) / args.steps
 
+    # rank-major ingest: the same steps as the gather delivers them (one
+    # [R][n][S] block per window), converted back into d in place of itself
+    def fill_gathered(x, out):
+        """out (flat) <- x [T][R][S] in the gather's layout, block by block."""
+        nfull, tail = w.T // w.W, w.T % w.W
+        n = nfull * w.W * w.R * w.S
+        out[:n].view(nfull, w.R, w.W, w.S).copy_(x[:nfull * w.W].view(nfull, w.W, w.R, w.S).permute(0, 2, 1, 3))
+        if tail:
+            out[n:].view(w.R, tail, w.S).copy_(x[nfull * w.W:].permute(1, 0, 2))
+        return out
+
+    g_dev = fill_gathered(d, torch.empty(w.T * w.R * w.S, dtype=torch.int64, device=device))
+    ingest_secs = timed_loop(lambda: sf.sf_gathered_to_steps(g_dev, w.T, w.R, w.S, w.W, dst=d), args.steps,
+                             args.warmup, ws, device, True) / args.steps
+    del g_dev
+
     # end to end through the host-memory entry point: every step streams the
     # pinned host tensor to the GPU in 2000-step chunks (copies overlapping the
     # previous chunk's compute) and reads the per-window results back
@@ -374,6 +390,21 @@ def run_ours(args):
     e2e_steps = max(3, args.steps // 2)
     e2e_secs = timed_loop(e2e_step, e2e_steps, args.warmup, ws, device, True)
     e2e_value = records * ws * e2e_steps / e2e_secs
+
+    # the same end to end over host telemetry in the gather's rank-major layout
+    g_host = fill_gathered(host, torch.empty(w.T * w.R * w.S, dtype=torch.int64, pin_memory=True))
+    gbufs = sf.StreamBuffers(w.T, w.R, w.S, w.W, w.k, chunk, device, gathered=True)
+
+    def e2e_gathered_step():
+        sf.sf_stream_gathered_windows(g_host, w.T, w.R, w.S, w.W, w.k, chunk, bufs=gbufs, status=pipe.status,
+                                      copy_stream=copy_stream)
+        for hb, o in zip(host_outs, [getattr(gbufs.out, n) for n in ("labels", "route_mask", "amb_mask", "share",
+                                                                      "gain", "top_stage", "top_pair",
+                                                                      "top_pair_value", "X", "D")]):
+            hb.copy_(o, non_blocking=True)
+
+    e2e_g_secs = timed_loop(e2e_gathered_step, e2e_steps, args.warmup, ws, device, True)
+    del gbufs, g_host
     if int(pipe.status.item()) != 0:
         raise RuntimeError("device status set during the end-to-end loop")
 
@@ -412,6 +443,11 @@ def run_ours(args):
         "group_pass": {"entry": "sf_group_aggregate", "groups": pipe.n_groups, "ms": round(group_secs * 1e3, 4),
                        "gbs": round(algo["group_aggregate"] / group_secs / 1e9, 1),
                        "frac": round(algo["group_aggregate"] / group_secs / 1e9 / peak, 4)},
+        "ingest_pass": {"entry": "sf_gathered_to_steps", "ms": round(ingest_secs * 1e3, 4),
+                        "gbs": round(2 * w.nbytes / ingest_secs / 1e9, 1),
+                        "frac": round(2 * w.nbytes / ingest_secs / 1e9 / peak, 4)},
+        "e2e_gathered": {"value": records * ws * e2e_steps / e2e_g_secs, "unit": UNIT,
+                         "entry": "sf_stream_gathered_windows", "h2d_bytes_per_step": w.nbytes},
         "gpu_launches": int(launches * args.steps // (args.steps + args.warmup)),
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": w.nbytes, "d2h_bytes_per_step": d2h,
                 "entry": "sf_stream_windows", "chunk_steps": chunk},

@@ -187,6 +187,17 @@ sf_status sf_stage_group_sum(const int64_t* X, int64_t nW, int64_t S, const int3
                              int64_t* Y, cudaStream_t stream);
 
 /*
+ * sf_gathered_to_steps - rank-major ingest.  The window-boundary gather of
+ * Sec. 5 leaves each window's telemetry as one [R][n][S] block (each rank's
+ * [n, S] buffer, in rank order).  This converts ceil(T / N) such blocks,
+ * stored one after another (block b holds steps b*N .. min(T, (b+1)*N) - 1,
+ * so only the last may be short), into the [T][R][S] layout every other
+ * entry point reads.  src and dst device, 16-byte aligned, not overlapping.
+ */
+sf_status sf_gathered_to_steps(const int64_t* src, int64_t T, int64_t R, int64_t S, int64_t N, int64_t* dst,
+                               cudaStream_t stream);
+
+/*
  * sf_topk_suspects - per window, the k stages with the largest X (Sec. 4
  * routing uses the top two shares) and the k (stage, rank) pairs with the
  * largest lead-rank credit E.  Order: value descending, then lower stage,
@@ -327,6 +338,24 @@ sf_status sf_stream_windows(const int64_t* h_d, int64_t T, int64_t R, int64_t S,
 
 /* Device staging bytes sf_stream_windows needs; 0 on bad arguments. */
 size_t sf_stream_windows_staging_size(int64_t T, int64_t R, int64_t S, int64_t chunk_steps);
+
+/*
+ * sf_stream_gathered_windows - sf_stream_windows over telemetry as the
+ * window-boundary gather delivers it (Sec. 5): h_g holds the windows'
+ * [R][n][S] blocks one after another (window w's block at element w*W*R*S,
+ * the last window possibly short), in host memory.  Each chunk is copied as
+ * is, converted on the device (sf_gathered_to_steps) into a third staging
+ * buffer, and then takes the same path.  Arguments and outputs as in
+ * sf_stream_windows; staging >= sf_stream_gathered_staging_size(...) bytes.
+ */
+sf_status sf_stream_gathered_windows(const int64_t* h_g, int64_t T, int64_t R, int64_t S, int64_t W, int32_t k,
+                                     int64_t chunk_steps, const sf_label_config* cfg, int64_t* staging,
+                                     size_t staging_bytes, void* workspace, size_t workspace_bytes, int64_t* X,
+                                     int64_t* Y, int64_t* D, int64_t* E, int32_t* C, int32_t* top_stage,
+                                     int32_t* top_pair, int64_t* top_pair_value, uint32_t* labels,
+                                     uint32_t* route_mask, uint32_t* amb_mask, double* share, double* gain,
+                                     uint32_t* status, cudaStream_t stream, cudaStream_t copy_stream);
+size_t sf_stream_gathered_staging_size(int64_t T, int64_t R, int64_t S, int64_t chunk_steps);
 
 /*
  * sf_label_windows_noalloc - sf_label_windows for callers that cannot

@@ -245,6 +245,16 @@ sf_status sf_stage_group_sum(const int64_t* X, int64_t nW, int64_t S, const int3
   return cuda_status(launch_stage_group_sum(X, nW, S, stage_group, K, Y, stream));
 }
 
+sf_status sf_gathered_to_steps(const int64_t* src, int64_t T, int64_t R, int64_t S, int64_t N, int64_t* dst,
+                               cudaStream_t stream) {
+  if (!src || !dst || !shape_ok(T, R, S) || N < 1) return SF_EINVAL;
+  const uintptr_t a = reinterpret_cast<uintptr_t>(src), b = reinterpret_cast<uintptr_t>(dst);
+  const uintptr_t bytes = uintptr_t(T) * uintptr_t(R) * uintptr_t(S) * 8u;
+  if (a < b + bytes && b < a + bytes) return SF_EINVAL;  // the copy is not in place
+  if (!aligned(src, 16) || !aligned(dst, 16)) return SF_EINVAL_ALIGN;
+  return cuda_status(launch_gathered_to_steps(src, T, R, S, N, dst, stream));
+}
+
 sf_status sf_topk_suspects(const int64_t* X, const int64_t* E, int64_t nW, int64_t S, int64_t R, int32_t k,
                            int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair,
                            int64_t* top_pair_value, cudaStream_t stream) {

@@ -65,6 +65,8 @@ cudaError_t launch_group_windows(const int64_t* d, int64_t T, int64_t R, int64_t
                                  cudaStream_t stream);
 cudaError_t launch_stage_group_sum(const int64_t* X, int64_t nW, int64_t S, const int32_t* stage_group, int64_t K,
                                    int64_t* Y, cudaStream_t stream);
+cudaError_t launch_gathered_to_steps(const int64_t* src, int64_t T, int64_t R, int64_t S, int64_t N, int64_t* dst,
+                                     cudaStream_t stream);
 cudaError_t launch_topk(const int64_t* X, const int64_t* E, int64_t nW, int64_t S, int64_t R,
                         int32_t k, int32_t* top_stage, int64_t* top_stage_value, int32_t* top_pair,
                         int64_t* top_pair_value, cudaStream_t stream);

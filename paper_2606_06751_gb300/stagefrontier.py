@@ -68,6 +68,9 @@ def _load():
                                      P, P, P, P, P, P, S],
         "sf_stream_windows": [P, I, I, I, I, I32, I, ctypes.POINTER(LabelConfig), P, ctypes.c_size_t, P,
                               ctypes.c_size_t, P, P, P, P, P, P, P, P, P, P, P, P, P, P, S, S],
+        "sf_stream_gathered_windows": [P, I, I, I, I, I32, I, ctypes.POINTER(LabelConfig), P, ctypes.c_size_t, P,
+                                       ctypes.c_size_t, P, P, P, P, P, P, P, P, P, P, P, P, P, P, S, S],
+        "sf_gathered_to_steps": [P, I, I, I, I, P, S],
     }
     for name, argt in sigs.items():
         f = getattr(L, name)
@@ -85,8 +88,9 @@ def _load():
     L.sf_label_config_default.restype = None
     L.sf_label_windows_workspace_size.argtypes = [I, I, I, I]
     L.sf_label_windows_workspace_size.restype = ctypes.c_size_t
-    L.sf_stream_windows_staging_size.argtypes = [I, I, I, I]
-    L.sf_stream_windows_staging_size.restype = ctypes.c_size_t
+    for name in ("sf_stream_windows_staging_size", "sf_stream_gathered_staging_size"):
+        getattr(L, name).argtypes = [I, I, I, I]
+        getattr(L, name).restype = ctypes.c_size_t
     return L
 
 
@@ -351,11 +355,13 @@ class Streamed:
 class StreamBuffers:
     """Device staging, workspace and outputs for sf_stream_windows, reusable across calls."""
 
-    def __init__(self, T: int, R: int, S: int, W: int, k: int, chunk_steps: int, device, lead_credit=True):
+    def __init__(self, T: int, R: int, S: int, W: int, k: int, chunk_steps: int, device, lead_credit=True,
+                 gathered=False):
         nW = (T + W - 1) // W
         e = lambda shape, dt: torch.empty(shape, dtype=dt, device=device)  # noqa: E731
         self.shape = (T, R, S, W, k, chunk_steps)
-        self.staging = e((int(_lib.sf_stream_windows_staging_size(T, R, S, chunk_steps)),), torch.uint8)
+        size = _lib.sf_stream_gathered_staging_size if gathered else _lib.sf_stream_windows_staging_size
+        self.staging = e((int(size(T, R, S, chunk_steps)),), torch.uint8)
         self.workspace = e((workspace_size(min(chunk_steps, T), R, S, W),), torch.uint8)
         self.out = Streamed(e((nW, S), torch.int64), e((nW, S), torch.int64), e((nW,), torch.int64),
                             e((nW, S, R), torch.int64) if lead_credit else None,
@@ -459,3 +465,34 @@ def sf_stage_group_sum(X, stage_group, K: int, Y=None, stream=None):
     Y = Y if Y is not None else _empty((nW, K), torch.int64, X)
     _check(_lib.sf_stage_group_sum(_p(X), nW, S, sg, K, _p(Y), _stream(stream)), "sf_stage_group_sum")
     return Y
+
+
+def sf_stream_gathered_windows(h_g: torch.Tensor, T: int, R: int, S: int, W: int, k: int, chunk_steps: int,
+                               bufs: StreamBuffers = None, cfg=None, status=None, stream=None,
+                               copy_stream=None) -> Streamed:
+    """h_g: int64 CPU tensor holding the windows' gathered [R][n][S] blocks one
+    after another (T*R*S values; pin it for copy/compute overlap)."""
+    if h_g.is_cuda or h_g.dtype != torch.int64 or not h_g.is_contiguous() or h_g.numel() != T * R * S:
+        raise TypeError("h_g must be a contiguous int64 host tensor of T*R*S values")
+    cfg = cfg if cfg is not None else default_config()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    if bufs is None:
+        bufs = StreamBuffers(T, R, S, W, k, chunk_steps, dev, gathered=True)
+    o = bufs.out
+    cs = copy_stream if copy_stream is not None else (stream if stream is not None else torch.cuda.current_stream())
+    _check(_lib.sf_stream_gathered_windows(h_g.data_ptr(), T, R, S, W, k, chunk_steps, ctypes.byref(cfg),
+                                           _p(bufs.staging), bufs.staging.numel(), _p(bufs.workspace),
+                                           bufs.workspace.numel(), _p(o.X), _p(o.Y), _p(o.D), _p(o.E), _p(o.C),
+                                           _p(o.top_stage), _p(o.top_pair), _p(o.top_pair_value), _p(o.labels),
+                                           _p(o.route_mask), _p(o.amb_mask), _p(o.share), _p(o.gain), _p(status),
+                                           _stream(stream), cs.cuda_stream), "sf_stream_gathered_windows")
+    return o
+
+
+def sf_gathered_to_steps(src: torch.Tensor, T: int, R: int, S: int, N: int, dst=None, stream=None):
+    """src: device int64 holding ceil(T/N) gathered [R][n][S] blocks; returns [T][R][S]."""
+    if not src.is_cuda or src.dtype != torch.int64 or not src.is_contiguous() or src.numel() != T * R * S:
+        raise TypeError("src must be a contiguous int64 CUDA tensor of T*R*S values")
+    dst = dst if dst is not None else torch.empty((T, R, S), dtype=torch.int64, device=src.device)
+    _check(_lib.sf_gathered_to_steps(_p(src), T, R, S, N, _p(dst), _stream(stream)), "sf_gathered_to_steps")
+    return dst

@@ -115,6 +115,10 @@ def test_host_validation(sf):
     sg = (ctypes.c_int32 * 4)(0, 1, 0, 1)
     assert L.sf_stage_group_sum(FAKE, 3, 4, sg, 33, FAKE, None) == sf.SF_EINVAL
     assert L.sf_stage_group_sum(FAKE + 4, 3, 4, sg, 2, FAKE, None) == sf.SF_EINVAL_ALIGN
+    # rank-major ingest: block length, in-place conversion, alignment
+    assert L.sf_gathered_to_steps(FAKE, 10, 4, 4, 0, FAKE + (1 << 16), None) == sf.SF_EINVAL
+    assert L.sf_gathered_to_steps(FAKE, 10, 4, 4, 5, FAKE + 64, None) == sf.SF_EINVAL
+    assert L.sf_gathered_to_steps(FAKE + 8, 10, 4, 4, 5, FAKE + (1 << 16), None) == sf.SF_EINVAL_ALIGN
     # nothing was launched by any of the rejected calls
     assert sf.launch_count() == 0
 
