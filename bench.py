@@ -233,6 +233,7 @@ class Pipeline:
                                  e((nW, S), torch.int64))
         self.lag = sf.Lag(e((T, S), torch.int64), e((T, S), torch.int64), e((T, S), torch.int64))
         self.spread = e((nW, S), torch.int64)
+        self.rank_ws = sf.rank_workspace(T, R, S, dev)
         # role groups: nodes of 128 consecutive ranks (one group when R <= 128)
         self.n_groups = max(1, R // 128)
         self.node_group = (torch.arange(R, device=dev, dtype=torch.int32) * self.n_groups // R).to(torch.int32)
@@ -273,11 +274,11 @@ class Pipeline:
 
     def rank_lag(self):
         """The cross-rank lag / delta-lag / gap pass (sf_rank_lag)."""
-        self.sf.sf_rank_lag(self.d, out=self.lag, status=self.status)
+        self.sf.sf_rank_lag(self.d, out=self.lag, workspace=self.rank_ws, status=self.status)
 
     def raw_spread(self):
         """The raw rank spread per window (sf_raw_spread)."""
-        self.sf.sf_raw_spread(self.d, self.w.W, spread=self.spread, status=self.status)
+        self.sf.sf_raw_spread(self.d, self.w.W, spread=self.spread, workspace=self.rank_ws, status=self.status)
 
     def group_aggregate(self):
         """The frontier within node groups of 128 ranks (sf_group_aggregate)."""

@@ -143,19 +143,27 @@ sf_status sf_window_baselines(const int64_t* d, int64_t T, int64_t R, int64_t S,
  *   dL [T][S] its increment L[t,s] - L[t,s-1] (L[t,-1] = 0),
  *   G  [T][S] max-minus-second-max gap F[t,s] - (second largest P[t,r,s]; a
  *             tie at the top counts as the second, so ties give 0; R = 1 gives 0).
- * Outputs device, nullable (at least one).
+ * Outputs device, nullable (at least one).  workspace: device, 256-byte
+ * aligned, at least one step's scratch; sf_rank_workspace_size(T, R, S)
+ * bytes (about 40 MB, so that the scratch stays in L2) processes the steps
+ * in the fewest chunks that still fit L2.  The workspace is overwritten and
+ * may be reused as soon as the call's work on `stream` is done.
  */
 sf_status sf_rank_lag(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t* L, int64_t* dL, int64_t* G,
-                      uint32_t* status, cudaStream_t stream);
+                      void* workspace, size_t workspace_bytes, uint32_t* status, cudaStream_t stream);
 
 /*
  * sf_raw_spread - the raw rank spread of the Sec. 6 routing table, per window
  * and stage: sum_t (max_r d[t,r,s] - median_r d[t,r,s]), lower median over
  * ranks.  spread [nW][S] device; windows, t0 and accumulate as in
- * sf_window_aggregate.
+ * sf_window_aggregate; workspace as in sf_rank_lag.
  */
 sf_status sf_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W,
-                        int64_t* spread, int32_t accumulate, uint32_t* status, cudaStream_t stream);
+                        int64_t* spread, int32_t accumulate, void* workspace, size_t workspace_bytes,
+                        uint32_t* status, cudaStream_t stream);
+
+/* Suggested workspace bytes for sf_rank_lag / sf_raw_spread (0 for a bad shape). */
+size_t sf_rank_workspace_size(int64_t T, int64_t R, int64_t S);
 
 /*
  * sf_group_aggregate - the frontier taken within role groups.  The App. A

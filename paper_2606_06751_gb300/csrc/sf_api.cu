@@ -201,22 +201,33 @@ sf_status sf_window_baselines(const int64_t* d, int64_t T, int64_t R, int64_t S,
 }
 
 sf_status sf_rank_lag(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t* L, int64_t* dL, int64_t* G,
-                      uint32_t* status, cudaStream_t stream) {
+                      void* workspace, size_t workspace_bytes, uint32_t* status, cudaStream_t stream) {
   if (!d || !shape_ok(T, R, S) || (!L && !dL && !G)) return SF_EINVAL;
-  if (!aligned(d, 16) || !aligned(L, 8) || !aligned(dL, 8) || !aligned(G, 8) || !aligned(status, 4))
+  if (!aligned(d, 16) || !aligned(L, 8) || !aligned(dL, 8) || !aligned(G, 8) || !aligned(status, 4) ||
+      !aligned(workspace, 256))
     return SF_EINVAL_ALIGN;
-  return cuda_status(launch_rank_select(d, T, R, S, 1, 0, 1, L, dL, G, nullptr, status, stream));
+  if (!workspace || !rank_workspace_ok(T, R, S, workspace_bytes)) return SF_EWORKSPACE;
+  return cuda_status(
+      launch_rank_select(d, T, R, S, 1, 0, 1, L, dL, G, nullptr, workspace, workspace_bytes, status, stream));
 }
 
 sf_status sf_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W, int64_t* spread,
-                        int32_t accumulate, uint32_t* status, cudaStream_t stream) {
+                        int32_t accumulate, void* workspace, size_t workspace_bytes, uint32_t* status,
+                        cudaStream_t stream) {
   if (!d || !spread || !shape_ok(T, R, S) || t0 < 0 || W < 1 || W > 65536 || (accumulate != 0 && accumulate != 1) ||
       t0 > (int64_t(1) << 62) - T)
     return SF_EINVAL;
-  if (!aligned(d, 16) || !aligned(spread, 8) || !aligned(status, 4)) return SF_EINVAL_ALIGN;
+  if (!aligned(d, 16) || !aligned(spread, 8) || !aligned(status, 4) || !aligned(workspace, 256))
+    return SF_EINVAL_ALIGN;
+  if (!workspace || !rank_workspace_ok(T, R, S, workspace_bytes)) return SF_EWORKSPACE;
   if (!accumulate && launch_zero(spread, size_t(sf_num_windows(t0, T, W)) * S * 8, stream) != cudaSuccess)
     return SF_ECUDA;
-  return cuda_status(launch_rank_select(d, T, R, S, 0, t0, W, nullptr, nullptr, nullptr, spread, status, stream));
+  return cuda_status(launch_rank_select(d, T, R, S, 0, t0, W, nullptr, nullptr, nullptr, spread, workspace,
+                                        workspace_bytes, status, stream));
+}
+
+size_t sf_rank_workspace_size(int64_t T, int64_t R, int64_t S) {
+  return shape_ok(T, R, S) ? rank_workspace_size(T, R, S) : 0;
 }
 
 sf_status sf_group_aggregate(const int64_t* d, int64_t T, int64_t R, int64_t S, const int32_t* group, int64_t G,

@@ -54,10 +54,10 @@ def _load():
         "sf_window_aggregate": [P, I, I, I, I, I, P, P, P, P, P, I32, P, S],
         "sf_topk_suspects": [P, P, I, I, I, I32, P, P, P, P, S],
         "sf_window_baselines": [P, I, I, I, I, I, P, P, P, P, I32, P, S],
-        "sf_rank_lag": [P, I, I, I, P, P, P, P, S],
+        "sf_rank_lag": [P, I, I, I, P, P, P, P, ctypes.c_size_t, P, S],
         "sf_group_aggregate": [P, I, I, I, P, I, I, I, P, P, I32, P, S],
         "sf_stage_group_sum": [P, I, I, P, I, P, S],
-        "sf_raw_spread": [P, I, I, I, I, I, P, I32, P, S],
+        "sf_raw_spread": [P, I, I, I, I, I, P, I32, P, ctypes.c_size_t, P, S],
         "sf_window_median": [P, I, I, I, I, P, P, S],
         "sf_direct_gain": [P, I, I, I, I, P, P, I32, Ratio, P, P, P, P, P, P, P, P, S],
         "sf_label_gates": [I, I, I, I, P, P, P, P, P, P, P, ctypes.POINTER(LabelConfig), P, P, P, P,
@@ -88,6 +88,8 @@ def _load():
     L.sf_label_config_default.restype = None
     L.sf_label_windows_workspace_size.argtypes = [I, I, I, I]
     L.sf_label_windows_workspace_size.restype = ctypes.c_size_t
+    L.sf_rank_workspace_size.argtypes = [I, I, I]
+    L.sf_rank_workspace_size.restype = ctypes.c_size_t
     for name in ("sf_stream_windows_staging_size", "sf_stream_gathered_staging_size"):
         getattr(L, name).argtypes = [I, I, I, I]
         getattr(L, name).restype = ctypes.c_size_t
@@ -423,20 +425,28 @@ class Lag:
     G: Optional[torch.Tensor]   # [T][S] max-minus-second-max gap
 
 
-def sf_rank_lag(d, out: Optional[Lag] = None, status=None, stream=None) -> Lag:
+def rank_workspace(T: int, R: int, S: int, device) -> torch.Tensor:
+    """Device scratch for sf_rank_lag / sf_raw_spread (reusable across calls)."""
+    return torch.empty(int(_lib.sf_rank_workspace_size(T, R, S)), dtype=torch.uint8, device=device)
+
+
+def sf_rank_lag(d, out: Optional[Lag] = None, workspace=None, status=None, stream=None) -> Lag:
     T, R, S = _d3(d)
     if out is None:
         out = Lag(_empty((T, S), torch.int64, d), _empty((T, S), torch.int64, d), _empty((T, S), torch.int64, d))
-    _check(_lib.sf_rank_lag(_p(d), T, R, S, _p(out.L), _p(out.dL), _p(out.G), _p(status), _stream(stream)),
-           "sf_rank_lag")
+    ws = workspace if workspace is not None else rank_workspace(T, R, S, d.device)
+    _check(_lib.sf_rank_lag(_p(d), T, R, S, _p(out.L), _p(out.dL), _p(out.G), _p(ws), ws.numel(), _p(status),
+                            _stream(stream)), "sf_rank_lag")
     return out
 
 
-def sf_raw_spread(d, W: int, t0: int = 0, spread=None, accumulate: bool = False, status=None, stream=None):
+def sf_raw_spread(d, W: int, t0: int = 0, spread=None, accumulate: bool = False, workspace=None, status=None,
+                  stream=None):
     T, R, S = _d3(d)
     spread = spread if spread is not None else _empty((num_windows(t0, T, W), S), torch.int64, d)
-    _check(_lib.sf_raw_spread(_p(d), T, R, S, t0, W, _p(spread), 1 if accumulate else 0, _p(status),
-                              _stream(stream)), "sf_raw_spread")
+    ws = workspace if workspace is not None else rank_workspace(T, R, S, d.device)
+    _check(_lib.sf_raw_spread(_p(d), T, R, S, t0, W, _p(spread), 1 if accumulate else 0, _p(ws), ws.numel(),
+                              _p(status), _stream(stream)), "sf_raw_spread")
     return spread
 
 

@@ -98,12 +98,17 @@ def test_host_validation(sf):
               None, None, None) == sf.SF_EINVAL_ALIGN
     assert L.sf_window_median(FAKE, 10, 4, 4, 0, FAKE, None, None) == sf.SF_EINVAL
     # cross-rank order statistics: no outputs, bad window, misaligned output
-    assert L.sf_rank_lag(FAKE, 10, 4, 4, None, None, None, None, None) == sf.SF_EINVAL
-    assert L.sf_rank_lag(FAKE, 10, 4, 4, FAKE + 4, None, None, None, None) == sf.SF_EINVAL_ALIGN
-    assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 0, FAKE, 0, None, None) == sf.SF_EINVAL
-    assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, None, 0, None, None) == sf.SF_EINVAL
-    assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, FAKE, 3, None, None) == sf.SF_EINVAL
-    assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, FAKE + 4, 0, None, None) == sf.SF_EINVAL_ALIGN
+    assert L.sf_rank_lag(FAKE, 10, 4, 4, None, None, None, FAKE, 1 << 20, None, None) == sf.SF_EINVAL
+    assert L.sf_rank_lag(FAKE, 10, 4, 4, FAKE + 4, None, None, FAKE, 1 << 20, None, None) == sf.SF_EINVAL_ALIGN
+    assert L.sf_rank_lag(FAKE, 10, 4, 4, FAKE, None, None, FAKE + 16, 1 << 20, None, None) == sf.SF_EINVAL_ALIGN
+    assert L.sf_rank_lag(FAKE, 10, 4, 4, FAKE, None, None, FAKE, 64, None, None) == sf.SF_EWORKSPACE
+    assert L.sf_rank_lag(FAKE, 10, 4, 4, FAKE, None, None, None, 1 << 20, None, None) == sf.SF_EWORKSPACE
+    assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 0, FAKE, 0, FAKE, 1 << 20, None, None) == sf.SF_EINVAL
+    assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, None, 0, FAKE, 1 << 20, None, None) == sf.SF_EINVAL
+    assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, FAKE, 3, FAKE, 1 << 20, None, None) == sf.SF_EINVAL
+    assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, FAKE + 4, 0, FAKE, 1 << 20, None, None) == sf.SF_EINVAL_ALIGN
+    assert L.sf_rank_workspace_size(8192, 8192, 8) >= 8 * 8192 * 4
+    assert L.sf_rank_workspace_size(0, 8, 8) == 0
     # role groups: group count, G*S limit, stage-group ids (host array)
     ga = L.sf_group_aggregate
     assert ga(FAKE, 10, 4, 4, FAKE, 0, 0, 5, FAKE, FAKE, 0, None, None) == sf.SF_EINVAL

@@ -73,10 +73,38 @@ def test_rank_lag_optional_outputs(sf):
     d_np = make(40, 33, 6, 5, "lognormal")
     o = O.rank_lag(d_np)
     d = dev(d_np)
-    only = sf.Lag(None, None, torch.empty((40, 6), dtype=torch.int64, device="cuda"))
-    sf.sf_rank_lag(d, out=only)
+    e = lambda: torch.empty((40, 6), dtype=torch.int64, device="cuda")  # noqa: E731
+    only_g = sf.sf_rank_lag(d, out=sf.Lag(None, None, e()))
+    only_dl = sf.sf_rank_lag(d, out=sf.Lag(None, e(), None))    # the lag is formed in dL and converted in place
+    l_dl = sf.sf_rank_lag(d, out=sf.Lag(e(), e(), None))
     torch.cuda.synchronize()
-    assert np.array_equal(host(only.G), o.G)
+    assert np.array_equal(host(only_g.G), o.G)
+    assert np.array_equal(host(only_dl.dL), o.dL)
+    assert np.array_equal(host(l_dl.L), o.L) and np.array_equal(host(l_dl.dL), o.dL)
+
+
+@pytest.mark.parametrize("T,R,S,steps_per_chunk", [(50, 100, 8, 1), (37, 1025, 6, 3), (12, 4096, 16, 5),
+                                                   (9, 7, 32, 2)])
+@pytest.mark.parametrize("kind", ["lognormal", "mixed"])
+def test_rank_lag_small_workspace_many_chunks(sf, T, R, S, steps_per_chunk, kind):
+    """A workspace that holds only a few steps: every chunk reuses the same
+    scratch (and its discarded L2 lines) for the next."""
+    d_np = make(T, R, S, T + R, kind)
+    o = O.rank_lag(d_np)
+    one = int(sf.lib().sf_rank_workspace_size(1, R, S))
+    ws = torch.empty(one * steps_per_chunk, dtype=torch.uint8, device="cuda")
+    g = sf.sf_rank_lag(dev(d_np), workspace=ws)
+    sp = sf.sf_raw_spread(dev(d_np), 4, t0=3, workspace=ws)
+    torch.cuda.synchronize()
+    assert np.array_equal(host(g.L), o.L) and np.array_equal(host(g.dL), o.dL) and np.array_equal(host(g.G), o.G)
+    assert np.array_equal(host(sp), O.raw_spread(d_np, 4, 3))
+
+
+def test_rank_lag_workspace_too_small_is_rejected(sf):
+    d = dev(make(4, 64, 8, 1, "lognormal"))
+    ws = torch.empty(256, dtype=torch.uint8, device="cuda")
+    with pytest.raises(RuntimeError):
+        sf.sf_rank_lag(d, workspace=ws)
 
 
 @pytest.mark.parametrize("T,R,S", [(20, 1, 1), (37, 3, 5), (301, 64, 4), (97, 40, 10), (1000, 8, 6),
