@@ -113,35 +113,71 @@ __device__ __forceinline__ void red_shared_inc_if(uint32_t* counter, bool pred) 
       : "memory");
 }
 
-// The k-th smallest of the live values among x[i] (row lane + 32 i), by byte
-// digits, most significant first.  Padding slots must hold 0xffffffff: they
-// sort after every live value (all below 2^nbits, or tying only at the top
-// when nbits = 32), so counting them never moves the rank-k bin and no slot
-// needs a validity test.  The first pass counts every slot; later passes
-// count, with a predicated increment, only values whose higher bytes match the
-// digits chosen so far.
-template <int NPL>
-__device__ __forceinline__ uint32_t warp_select_bytes32(const uint32_t (&x)[NPL], int nbits, uint32_t k,
-                                                        uint32_t* hist, int lane) {
-  uint32_t prefix = 0, himask = 0, rem = k;
-  for (int b = (nbits + 7) / 8 - 1; b >= 0; --b) {
+// The k-th smallest of the live values among x[i] (row lane + 32 i), all
+// below 2^nbits.  Padding slots must hold 2^nbits - 1: they sort at or after
+// every live value, so counting them never moves the rank-k bin and no slot
+// needs a validity test.  The first digit takes the top 8 bits of the range,
+// [nbits - 8, nbits), so it spreads over the 256 bins and its chosen bin
+// usually holds a few percent of the column; the next pass then keeps the
+// values of that bin as candidates (in this warp's own, already consumed
+// column slots of the tile: slot j at cand(j)) and every later pass reads only
+// those.  A bin too full to keep (heavy ties) falls back to predicated
+// increments over all slots.
+template <int NPL, typename CandAddr>
+__device__ __forceinline__ uint32_t warp_select_bits32(const uint32_t (&x)[NPL], int nbits, uint32_t k,
+                                                       uint32_t* hist, int lane, CandAddr cand) {
+  constexpr uint32_t kCap = 32u * NPL < 512u ? 32u * NPL : 512u;  // candidate slots
+  if (nbits == 0) return 0;
+  int sh = nbits > 8 ? nbits - 8 : 0;
+  reinterpret_cast<uint4*>(hist)[2 * lane] = make_uint4(0, 0, 0, 0);
+  reinterpret_cast<uint4*>(hist)[2 * lane + 1] = make_uint4(0, 0, 0, 0);
+  __syncwarp();
+#pragma unroll
+  for (int i = 0; i < NPL; ++i) atomicAdd(&hist[x[i] >> sh], 1u);  // x < 2^nbits: the bin is below 256
+  __syncwarp();
+  uint32_t digit, below;
+  hist_find(hist, k, lane, digit, below);
+  uint32_t rem = k - below;
+  uint32_t prefix = digit << sh;
+  const uint32_t kept = hist[digit];  // values the next pass matches
+  int hi = sh;                        // offset bits at and above hi are chosen
+  if (hi == 0) return prefix;
+  uint32_t* ncand = hist + 256;  // spare word after the bins
+  const bool compact = kept <= kCap;
+  bool keep_pass = compact;  // the next pass keeps the candidates
+  __syncwarp();
+  while (hi > 0) {
+    sh = hi > 8 ? hi - 8 : 0;
+    const uint32_t mask = (1u << (hi - sh)) - 1u;
     reinterpret_cast<uint4*>(hist)[2 * lane] = make_uint4(0, 0, 0, 0);
     reinterpret_cast<uint4*>(hist)[2 * lane + 1] = make_uint4(0, 0, 0, 0);
+    if (lane == 0) *ncand = 0;
     __syncwarp();
-    const uint32_t sel = 0x4440u | uint32_t(b);  // __byte_perm selector: byte b of x, zero above
-    if (himask == 0) {
+    if (!compact) {
 #pragma unroll
-      for (int i = 0; i < NPL; ++i) atomicAdd(&hist[__byte_perm(x[i], 0, sel)], 1u);
+      for (int i = 0; i < NPL; ++i)
+        red_shared_inc_if(&hist[(x[i] >> sh) & mask], (x[i] >> hi) == (prefix >> hi));
+    } else if (keep_pass) {
+      // the pass after the first: count and keep the matching values
+#pragma unroll
+      for (int i = 0; i < NPL; ++i) {
+        if ((x[i] >> hi) == (prefix >> hi)) {
+          atomicAdd(&hist[(x[i] >> sh) & mask], 1u);
+          *cand(atomicAdd(ncand, 1u)) = x[i];
+        }
+      }
     } else {
-#pragma unroll
-      for (int i = 0; i < NPL; ++i) red_shared_inc_if(&hist[__byte_perm(x[i], 0, sel)], (x[i] & himask) == prefix);
+      for (uint32_t j = lane; j < kept; j += 32) {
+        const uint32_t v = *cand(j);
+        red_shared_inc_if(&hist[(v >> sh) & mask], (v >> hi) == (prefix >> hi));
+      }
     }
     __syncwarp();
-    uint32_t digit, below;
     hist_find(hist, rem, lane, digit, below);
     rem -= below;
-    prefix |= digit << (8 * b);
-    himask |= 0xffu << (8 * b);
+    prefix |= digit << sh;
+    hi = sh;
+    keep_pass = false;
     __syncwarp();
   }
   return prefix;
@@ -298,9 +334,15 @@ __global__ void __launch_bounds__(kMedThreads, 3)
     lmax = __reduce_max_sync(kFull, lmax);
     const uint32_t range = lmax - lmin;
     const int nbits = range ? 32 - __clz(static_cast<int>(range)) : 0;
+    const uint32_t pad = nbits == 32 ? 0xffffffffu : (1u << nbits) - 1u;  // sorts at or after every live value
 #pragma unroll
-    for (int i = 0; i < NPL; ++i) xl[i] = 32 * i < live ? xl[i] - lmin : 0xffffffffu;
-    const uint32_t ans = warp_select_bytes32<NPL>(xl, nbits, k, hist, lane);
+    for (int i = 0; i < NPL; ++i) xl[i] = 32 * i < live ? xl[i] - lmin : pad;
+    // candidate slot j: this warp's (already consumed) column slot of tile row j
+    const uint32_t swz = (warp & 1) << 3;
+    auto cand = [&](uint32_t j) {
+      return reinterpret_cast<uint32_t*>(tile + j * 64u + ((((warp >> 1) ^ ((j >> 1) & 3u)) << 4) | swz));
+    };
+    const uint32_t ans = warp_select_bits32<NPL>(xl, nbits, k, hist, lane, cand);
     key = (static_cast<uint64_t>(hmin) << 32) | (lmin + ans);
   } else {
     constexpr uint64_t kSign = 1ull << 63;

@@ -112,6 +112,17 @@ def _stream(stream) -> int:
     return s.cuda_stream
 
 
+def _hold(tensors, *streams):
+    """Temporaries the binding allocated for work enqueued on `streams`: the
+    caching allocator may reuse their memory only once that work is done."""
+    cur = torch.cuda.current_stream()
+    for st in streams:
+        if st is not None and st != cur:
+            for t in tensors:
+                if t is not None:
+                    t.record_stream(st)
+
+
 def _check(rc: int, where: str):
     if rc != SF_OK:
         raise SFError(rc, where)
@@ -304,6 +315,7 @@ def sf_label_windows(d, W: int, role=None, missing=None, wall=None, other_stage:
     need = workspace_size(T, R, S, W)
     if workspace is None:
         workspace = torch.empty(need, dtype=torch.uint8, device=d.device)
+        _hold([workspace], stream)
     if out is None:
         out = _label_out(nW, S, d)
         if evidence:
@@ -382,10 +394,12 @@ def sf_stream_windows(h_d: torch.Tensor, W: int, k: int, chunk_steps: int, bufs:
     T, R, S = h_d.shape
     cfg = cfg if cfg is not None else default_config()
     dev = torch.device("cuda", torch.cuda.current_device())
-    if bufs is None:
-        bufs = StreamBuffers(T, R, S, W, k, chunk_steps, dev)
-    o = bufs.out
     cs = copy_stream if copy_stream is not None else (stream if stream is not None else torch.cuda.current_stream())
+    if bufs is None:
+        # staging and workspace are used by both streams: keep them until that work is done
+        bufs = StreamBuffers(T, R, S, W, k, chunk_steps, dev)
+        _hold([bufs.staging, bufs.workspace], cs, stream)
+    o = bufs.out
     _check(_lib.sf_stream_windows(h_d.data_ptr(), T, R, S, W, k, chunk_steps, ctypes.byref(cfg),
                                   _p(bufs.staging), bufs.staging.numel(), _p(bufs.workspace), bufs.workspace.numel(),
                                   _p(o.X), _p(o.Y), _p(o.D), _p(o.E), _p(o.C), _p(o.top_stage), _p(o.top_pair),
@@ -434,7 +448,10 @@ def sf_rank_lag(d, out: Optional[Lag] = None, workspace=None, status=None, strea
     T, R, S = _d3(d)
     if out is None:
         out = Lag(_empty((T, S), torch.int64, d), _empty((T, S), torch.int64, d), _empty((T, S), torch.int64, d))
-    ws = workspace if workspace is not None else rank_workspace(T, R, S, d.device)
+    ws = workspace
+    if ws is None:
+        ws = rank_workspace(T, R, S, d.device)
+        _hold([ws], stream)
     _check(_lib.sf_rank_lag(_p(d), T, R, S, _p(out.L), _p(out.dL), _p(out.G), _p(ws), ws.numel(), _p(status),
                             _stream(stream)), "sf_rank_lag")
     return out
@@ -444,7 +461,10 @@ def sf_raw_spread(d, W: int, t0: int = 0, spread=None, accumulate: bool = False,
                   stream=None):
     T, R, S = _d3(d)
     spread = spread if spread is not None else _empty((num_windows(t0, T, W), S), torch.int64, d)
-    ws = workspace if workspace is not None else rank_workspace(T, R, S, d.device)
+    ws = workspace
+    if ws is None:
+        ws = rank_workspace(T, R, S, d.device)
+        _hold([ws], stream)
     _check(_lib.sf_raw_spread(_p(d), T, R, S, t0, W, _p(spread), 1 if accumulate else 0, _p(ws), ws.numel(),
                               _p(status), _stream(stream)), "sf_raw_spread")
     return spread
@@ -486,10 +506,11 @@ def sf_stream_gathered_windows(h_g: torch.Tensor, T: int, R: int, S: int, W: int
         raise TypeError("h_g must be a contiguous int64 host tensor of T*R*S values")
     cfg = cfg if cfg is not None else default_config()
     dev = torch.device("cuda", torch.cuda.current_device())
+    cs = copy_stream if copy_stream is not None else (stream if stream is not None else torch.cuda.current_stream())
     if bufs is None:
         bufs = StreamBuffers(T, R, S, W, k, chunk_steps, dev, gathered=True)
+        _hold([bufs.staging, bufs.workspace], cs, stream)
     o = bufs.out
-    cs = copy_stream if copy_stream is not None else (stream if stream is not None else torch.cuda.current_stream())
     _check(_lib.sf_stream_gathered_windows(h_g.data_ptr(), T, R, S, W, k, chunk_steps, ctypes.byref(cfg),
                                            _p(bufs.staging), bufs.staging.numel(), _p(bufs.workspace),
                                            bufs.workspace.numel(), _p(o.X), _p(o.Y), _p(o.D), _p(o.E), _p(o.C),

@@ -152,11 +152,18 @@ def test_topk_parity(sf, nW, S, R, k):
 @pytest.mark.parametrize("T,R,S,W", [(100, 8, 6, 100), (250, 4, 3, 32), (130, 5, 4, 64), (300, 2, 8, 128),
                                      (700, 3, 2, 256), (1100, 2, 4, 512), (2100, 1, 4, 1000),
                                      (2200, 2, 2, 1024), (2500, 1, 3, 1100), (45, 1024, 10, 20)])
-@pytest.mark.parametrize("kind", ["ties", "lognormal", "wide"])
+@pytest.mark.parametrize("kind", ["ties", "lognormal", "wide", "zeros", "ranges", "clusters"])
 def test_median_parity(sf, T, R, S, W, kind):
+    rng = np.random.default_rng(T + W)
     if kind == "wide":  # signed values spanning more than 2^32: the 64-bit search path
-        rng = np.random.default_rng(T + W)
         d_np = rng.integers(-(1 << 40), 1 << 40, size=(T, R, S), dtype=np.int64)
+    elif kind == "ranges":  # per-column range from 1 to 32 bits (the last at the 32-bit edge)
+        bits = rng.integers(0, 33, size=(1, R, S))
+        bits[0, 0, 0] = 32
+        d_np = (rng.integers(0, 1 << 62, size=(T, R, S), dtype=np.int64) % (np.int64(1) << bits)) + (1 << 33)
+    elif kind == "clusters":  # a few tight clusters: the chosen top-digit bin is large or just fits
+        centers = rng.integers(0, 1 << 30, size=(4,))
+        d_np = centers[rng.integers(0, 4, size=(T, R, S))] + rng.integers(0, 3, size=(T, R, S))
     else:
         d_np = make(T, R, S, T + W, kind)
     o = O.window_median(d_np, W)
