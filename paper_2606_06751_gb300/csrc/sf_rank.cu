@@ -4,7 +4,8 @@
 // with the maximum and the second largest value.
 //
 // The steps are processed in chunks whose scratch stays in L2; per chunk two
-// kernels run back to back:
+// kernels run, the encode of the next chunk overlapping the select of this
+// one (programmatic dependent launch, two scratch buffers):
 //  rank_encode_kernel - streams the chunk's rank rows once from HBM (16-byte
 //    loads, two rows in flight per thread, the stage prefix in registers) and
 //    writes every (step, stage)
@@ -37,7 +38,7 @@ constexpr int kEncRows = 2048;  // rank rows per encode item (8 per thread)
 constexpr int kSelThreads = 256;
 constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kSelCand = 2048;  // candidate keys a column may keep after the second pass
-constexpr size_t kRkChunkTarget = size_t(64) << 20;  // scratch of one chunk, inside L2
+constexpr size_t kRkChunkTarget = size_t(40) << 20;  // scratch of one chunk buffer; two fit L2
 
 struct RankParams {
   const int64_t* d;
@@ -72,6 +73,12 @@ __device__ __forceinline__ void top2_merge(V& a1, V& a2, V b1, V b2) {
 __device__ __forceinline__ int64_t key_value(int64_t ref, uint32_t key) {
   return ref + static_cast<int64_t>(static_cast<int32_t>(key ^ 0x80000000u));
 }
+
+// Programmatic dependent launch: the encode of chunk c+1 runs while the
+// select of chunk c does; each kernel waits for its predecessor in the stream
+// only where it must (see launch_rank_select).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 __device__ __forceinline__ void discard_l2_line(const void* p) {
   asm volatile("discard.global.L2 [%0], 128;" ::"l"(p) : "memory");
@@ -203,6 +210,11 @@ __global__ void __launch_bounds__(kEncThreads) rank_encode_kernel(const RankPara
   }
   const uint32_t bits = range_bits(__reduce_or_sync(kFull, dor), p.of_prefix ? __reduce_or_sync(kFull, tor) : 0u);
   if (lane == 0) report(p.status, bits);
+  // let this chunk's select launch, then finish only once the previous
+  // chunk's select (which read the other scratch buffer) has finished, so
+  // that this kernel's completion implies every earlier kernel's
+  pdl_launch_dependents();
+  pdl_wait();
 }
 
 // ------------------------------------------------------------------ select
@@ -302,6 +314,10 @@ __global__ void __launch_bounds__(kSelThreads, 6) rank_select_kernel(const RankP
   const int S = static_cast<int>(p.S);
   const int R = static_cast<int>(p.R);
   const int64_t tasks = p.Tc * S;
+  // this chunk's encode (and, through its own wait, every earlier kernel) is
+  // complete and visible; then the next chunk's encode may start
+  pdl_wait();
+  pdl_launch_dependents();
   for (int64_t task = blockIdx.x; task < tasks; task += gridDim.x) {
     const int64_t tl = task / S;
     const int s = static_cast<int>(task - tl * S);
@@ -502,6 +518,20 @@ int64_t chunk_steps_for(int64_t T, int64_t R, int64_t S, size_t bytes) {
   return lo;
 }
 
+template <typename K>
+cudaError_t launch_pdl(K kern, int grid, int threads, const RankParams& p, cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = dim3(static_cast<unsigned>(grid));
+  cfg.blockDim = dim3(static_cast<unsigned>(threads));
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, p);
+}
+
 template <int SC>
 cudaError_t launch_encode(const RankParams& p, cudaStream_t stream) {
   static int per_sm = 0;  // resident CTAs per SM (same on every GB300)
@@ -512,28 +542,33 @@ cudaError_t launch_encode(const RankParams& p, cudaStream_t stream) {
     per_sm = 1;
   }
   const int grid = static_cast<int>(std::min<int64_t>(p.Tc * p.nblk, int64_t(per_sm) * sm_count()));
-  rank_encode_kernel<SC><<<grid, kEncThreads, 0, stream>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(rank_encode_kernel<SC>, grid, kEncThreads, p, stream);
 }
 
 }  // namespace
 
+// The workspace holds two chunk buffers: the encode of chunk c+1 fills one
+// while the select of chunk c reads the other.
 size_t rank_workspace_size(int64_t T, int64_t R, int64_t S) {
   if (T < 1 || R < 1 || S < 1) return 0;
   const size_t one = layout_for(R, S, 1).total;
   const int64_t want = std::max<int64_t>(1, std::min<int64_t>(T, int64_t(kRkChunkTarget / one)));
-  return layout_for(R, S, want).total;
+  return 2 * layout_for(R, S, want).total;
 }
 
-bool rank_workspace_ok(int64_t T, int64_t R, int64_t S, size_t bytes) { return chunk_steps_for(T, R, S, bytes) > 0; }
+bool rank_workspace_ok(int64_t T, int64_t R, int64_t S, size_t bytes) {
+  return chunk_steps_for(T, R, S, bytes / 2 & ~size_t(255)) > 0;
+}
 
 cudaError_t launch_rank_select(const int64_t* d, int64_t T, int64_t R, int64_t S, int of_prefix, int64_t t0,
                                int64_t W, int64_t* L, int64_t* dL, int64_t* G, int64_t* spread, void* workspace,
                                size_t ws_bytes, uint32_t* status, cudaStream_t stream) {
-  const int64_t Tc = chunk_steps_for(T, R, S, ws_bytes);
+  const size_t half = ws_bytes / 2 & ~size_t(255);  // one chunk buffer, 256-byte aligned
+  const int64_t Tc = chunk_steps_for(T, R, S, half);
   if (Tc < 1) return cudaErrorInvalidValue;
   const ScratchLayout l = layout_for(R, S, Tc);
-  unsigned char* ws = static_cast<unsigned char*>(workspace);
+  unsigned char* const ws_base = static_cast<unsigned char*>(workspace);
+  unsigned char* ws = ws_base;
   RankParams p{};
   p.d = d;
   p.T = T;
@@ -556,9 +591,16 @@ cudaError_t launch_rank_select(const int64_t* d, int64_t T, int64_t R, int64_t S
   p.pbad = reinterpret_cast<uint32_t*>(ws + l.pbad);
   p.ref = reinterpret_cast<int64_t*>(ws + l.ref);
   const int sms = sm_count();
-  for (int64_t c0 = 0; c0 < T; c0 += Tc) {
+  for (int64_t c0 = 0, c = 0; c0 < T; c0 += Tc, ++c) {
     p.c0 = c0;
     p.Tc = std::min(Tc, T - c0);
+    ws = ws_base + (c & 1) * half;  // alternate the two chunk buffers
+    p.keys = reinterpret_cast<uint32_t*>(ws + l.keys);
+    p.pmin = reinterpret_cast<uint32_t*>(ws + l.pmin);
+    p.pmax = reinterpret_cast<uint32_t*>(ws + l.pmax);
+    p.psec = reinterpret_cast<uint32_t*>(ws + l.psec);
+    p.pbad = reinterpret_cast<uint32_t*>(ws + l.pbad);
+    p.ref = reinterpret_cast<int64_t*>(ws + l.ref);
     count_launch();
     cudaError_t e;
     switch (S) {
@@ -572,8 +614,7 @@ cudaError_t launch_rank_select(const int64_t* d, int64_t T, int64_t R, int64_t S
     if (e != cudaSuccess) return e;
     const int sel_grid = static_cast<int>(std::min<int64_t>(p.Tc * S, int64_t(sms) * 6));
     count_launch();
-    rank_select_kernel<<<sel_grid, kSelThreads, 0, stream>>>(p);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = launch_pdl(rank_select_kernel, sel_grid, kSelThreads, p, stream)) != cudaSuccess) return e;
   }
   if (of_prefix && dL) {
     const int grid = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>((T + 255) / 256, int64_t(sms) * 4)));
