@@ -121,7 +121,8 @@ __device__ __forceinline__ void red_shared_inc_if(uint32_t* counter, bool pred) 
 // usually holds a few percent of the column; the next pass then keeps the
 // values of that bin as candidates (in this warp's own, already consumed
 // column slots of the tile: slot j at cand(j)) and every later pass reads only
-// those.  A bin too full to keep (heavy ties) falls back to predicated
+// those; a bin of at most 32 values is finished directly, one value per lane,
+// by counting.  A bin too full to keep (heavy ties) falls back to predicated
 // increments over all slots.
 template <int NPL, typename CandAddr>
 __device__ __forceinline__ uint32_t warp_select_bits32(const uint32_t (&x)[NPL], int nbits, uint32_t k,
@@ -143,6 +144,31 @@ __device__ __forceinline__ uint32_t warp_select_bits32(const uint32_t (&x)[NPL],
   int hi = sh;                        // offset bits at and above hi are chosen
   if (hi == 0) return prefix;
   uint32_t* ncand = hist + 256;  // spare word after the bins
+  if (kept <= 32) {
+    // at most one value of the chosen bin per lane: gather them and take the
+    // rem-th smallest by counting, instead of more histogram passes
+    __syncwarp();
+    if (lane == 0) *ncand = 0;
+    __syncwarp();
+#pragma unroll
+    for (int i = 0; i < NPL; ++i)
+      if ((x[i] >> hi) == digit) *cand(atomicAdd(ncand, 1u)) = x[i];
+    __syncwarp();
+    const bool mine = static_cast<uint32_t>(lane) < kept;
+    const uint32_t v = mine ? *cand(lane) : 0u;
+    uint32_t lt = 0, le = 0;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const uint32_t c = __shfl_sync(kFull, v, j);
+      const bool live = static_cast<uint32_t>(j) < kept;
+      lt += (live && c < v) ? 1u : 0u;
+      le += (live && c <= v) ? 1u : 0u;
+    }
+    const uint32_t hit = __ballot_sync(kFull, mine && lt <= rem && rem < le);
+    const uint32_t ans = __shfl_sync(kFull, v, __ffs(hit) - 1);
+    __syncwarp();
+    return ans;
+  }
   const bool compact = kept <= kCap;
   bool keep_pass = compact;  // the next pass keeps the candidates
   __syncwarp();
