@@ -35,7 +35,7 @@ namespace {
 constexpr int kRkMaxS = 32;
 constexpr int kEncThreads = 256;
 constexpr int kEncRows = 2048;  // rank rows per encode item (8 per thread)
-constexpr int kSelThreads = 256;
+constexpr int kSelThreads = 128;
 constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kSelCand = 2048;  // candidate keys a column may keep after the second pass
 constexpr size_t kRkChunkTarget = size_t(40) << 20;  // scratch of one chunk buffer; two fit L2
@@ -217,6 +217,130 @@ __global__ void __launch_bounds__(kEncThreads) rank_encode_kernel(const RankPara
   pdl_wait();
 }
 
+// Encode with a rank row split over SC/2 lanes (SC = 4, 8 or 16): lane j of a
+// group holds stages 2j and 2j+1 (one 16-byte load), the stage prefix comes
+// from a segmented warp scan of the pair sums, and each thread keeps the
+// statistics of its two columns only.  Few registers per thread let many
+// CTAs, and four loads per thread, be in flight on each SM.
+template <int SC>
+__global__ void __launch_bounds__(kEncThreads) rank_encode_split_kernel(const RankParams p) {
+  constexpr int L = SC / 2;                     // lanes per rank row
+  constexpr int kRowsPerPass = kEncThreads / L;  // rows the CTA covers per pass
+  constexpr int kUnroll = 4;                     // passes whose loads are in flight together
+  constexpr int kWarps = kEncThreads / 32;
+  __shared__ int64_t sref[kRkMaxS];
+  __shared__ uint32_t wmn[kWarps][kRkMaxS], wmx[kWarps][kRkMaxS], wm2[kWarps][kRkMaxS];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int j = lane % L;                      // this thread's stage pair
+  const int rsub = tid / L;                    // this thread's row within a pass
+  const int64_t R = p.R;
+  uint32_t dor = 0, tor = 0;
+  const int64_t items = p.Tc * p.nblk;
+  for (int64_t item = blockIdx.x; item < items; item += gridDim.x) {
+    const int64_t tl = item / p.nblk;
+    const int blk = static_cast<int>(item - tl * p.nblk);
+    const int64_t* dt = p.d + (p.c0 + tl) * R * SC;
+    if (warp == 0) {
+      int64_t x = lane < SC ? __ldg(dt + lane) : 0;
+      if (p.of_prefix) {
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int64_t up = __shfl_up_sync(kFull, x, o);
+          if (lane >= o) x += up;
+        }
+      }
+      if (lane < SC) {
+        sref[lane] = x;
+        if (blk == 0) p.ref[tl * SC + lane] = x;
+      }
+    }
+    __syncthreads();
+    const int64_t ref0 = sref[2 * j], ref1 = sref[2 * j + 1];
+    uint32_t mn0 = 0xffffffffu, a0 = 0u, b0 = 0u, mn1 = 0xffffffffu, a1 = 0u, b1 = 0u;
+    bool bad = false;
+    const int64_t rb = int64_t(blk) * kEncRows;
+    const int nrows = static_cast<int>(R - rb < kEncRows ? R - rb : kEncRows);
+    uint32_t* k0 = p.keys + (tl * SC + 2 * j) * p.ldR + rb;
+    uint32_t* k1 = k0 + p.ldR;
+    const longlong2* base = reinterpret_cast<const longlong2*>(dt + rb * SC) + j;
+    for (int r0 = 0; r0 < nrows; r0 += kUnroll * kRowsPerPass) {
+      longlong2 v[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int r = r0 + u * kRowsPerPass + rsub;
+        v[u] = r < nrows ? __ldg(base + int64_t(r) * L) : make_longlong2(0, 0);
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int r = r0 + u * kRowsPerPass + rsub;
+        const bool live = r < nrows;
+        dor |= static_cast<uint32_t>(static_cast<uint64_t>(v[u].x) >> 32) |
+               static_cast<uint32_t>(static_cast<uint64_t>(v[u].y) >> 32);
+        int64_t x0 = v[u].x, x1 = v[u].y;
+        if (p.of_prefix) {
+          // prefix before this pair: scan of the pair sums over the row's lanes
+          const int64_t pair = x0 + x1;
+          int64_t incl = pair;
+#pragma unroll
+          for (int o = 1; o < L; o <<= 1) {
+            const int64_t up = __shfl_up_sync(kFull, incl, o, L);
+            if (j >= o) incl += up;
+          }
+          x0 += incl - pair;
+          x1 = incl;
+          if (j == L - 1) tor |= static_cast<uint32_t>(static_cast<uint64_t>(incl) >> 32);
+        }
+        const int64_t d0 = x0 - ref0, d1 = x1 - ref1;
+        const uint32_t q0 = static_cast<uint32_t>(d0) ^ 0x80000000u, q1 = static_cast<uint32_t>(d1) ^ 0x80000000u;
+        if (live) {
+          bad |= ((static_cast<uint64_t>(d0 + 0x80000000ll) | static_cast<uint64_t>(d1 + 0x80000000ll)) >> 32) != 0;
+          k0[r] = q0;
+          k1[r] = q1;
+          mn0 = q0 < mn0 ? q0 : mn0;
+          mn1 = q1 < mn1 ? q1 : mn1;
+          top2_merge<uint32_t>(a0, b0, q0, 0u);
+          top2_merge<uint32_t>(a1, b1, q1, 0u);
+        }
+      }
+    }
+    // merge the lanes of equal j (offsets that are multiples of L), then the warps
+#pragma unroll
+    for (int o = L; o < 32; o <<= 1) {
+      mn0 = min(mn0, __shfl_xor_sync(kFull, mn0, o));
+      mn1 = min(mn1, __shfl_xor_sync(kFull, mn1, o));
+      const uint32_t oa0 = __shfl_xor_sync(kFull, a0, o), ob0 = __shfl_xor_sync(kFull, b0, o);
+      const uint32_t oa1 = __shfl_xor_sync(kFull, a1, o), ob1 = __shfl_xor_sync(kFull, b1, o);
+      top2_merge<uint32_t>(a0, b0, oa0, ob0);
+      top2_merge<uint32_t>(a1, b1, oa1, ob1);
+    }
+    if (lane < L) {
+      wmn[warp][2 * j] = mn0;
+      wmx[warp][2 * j] = a0;
+      wm2[warp][2 * j] = b0;
+      wmn[warp][2 * j + 1] = mn1;
+      wmx[warp][2 * j + 1] = a1;
+      wm2[warp][2 * j + 1] = b1;
+    }
+    const int any_bad = __syncthreads_or(bad ? 1 : 0);
+    if (tid < SC) {
+      uint32_t a = wmn[0][tid], x1 = wmx[0][tid], x2 = wm2[0][tid];
+      for (int w = 1; w < kWarps; ++w) {
+        a = wmn[w][tid] < a ? wmn[w][tid] : a;
+        top2_merge<uint32_t>(x1, x2, wmx[w][tid], wm2[w][tid]);
+      }
+      p.pmin[item * SC + tid] = a;
+      p.pmax[item * SC + tid] = x1;
+      p.psec[item * SC + tid] = x2;
+    }
+    if (tid == 0) p.pbad[item] = static_cast<uint32_t>(any_bad);
+    __syncthreads();  // sref and the warp partials are rewritten by the next item
+  }
+  const uint32_t bits = range_bits(__reduce_or_sync(kFull, dor), p.of_prefix ? __reduce_or_sync(kFull, tor) : 0u);
+  if (lane == 0) report(p.status, bits);
+  pdl_launch_dependents();
+  pdl_wait();
+}
+
 // ------------------------------------------------------------------ select
 
 struct SelShared {
@@ -283,7 +407,7 @@ __device__ __noinline__ void select_column_64(const RankParams& p, int64_t t, in
   }
   __syncthreads();
   for (int bb = sh.bytes64 - 1; bb >= 0; --bb) {
-    sh.hist[tid] = 0;
+    for (int i = tid; i < 256; i += kSelThreads) sh.hist[i] = 0;
     __syncthreads();
     const int shift = 8 * bb;
     const int64_t lo = sh.lo64;
@@ -308,7 +432,7 @@ __device__ __noinline__ void select_column_64(const RankParams& p, int64_t t, in
   __syncthreads();
 }
 
-__global__ void __launch_bounds__(kSelThreads, 6) rank_select_kernel(const RankParams p) {
+__global__ void __launch_bounds__(kSelThreads, 12) rank_select_kernel(const RankParams p) {
   __shared__ __align__(16) SelShared sh;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int S = static_cast<int>(p.S);
@@ -361,7 +485,7 @@ __global__ void __launch_bounds__(kSelThreads, 6) rank_select_kernel(const RankP
       const int nb = sh.nb;
       // ---- first pass: every key counts (the top digit), four keys per load
       if (nb > 0) {
-        sh.hist[tid] = 0;
+        for (int i = tid; i < 256; i += kSelThreads) sh.hist[i] = 0;
         __syncthreads();
         const int shift = nb > 8 ? nb - 8 : 0;  // offsets are below 2^nb: no mask needed
         const int nq = R >> 2;
@@ -392,7 +516,7 @@ __global__ void __launch_bounds__(kSelThreads, 6) rank_select_kernel(const RankP
         __syncthreads();  // the last digit search is done: its pref and rem are visible, hist is free
         const uint32_t pref = sh.pref;
         const bool compact = sh.compact != 0;
-        sh.hist[tid] = 0;
+        for (int i = tid; i < 256; i += kSelThreads) sh.hist[i] = 0;
         __syncthreads();
         if (read_all) {
           // second pass: count the matching keys; keep them when they are few
@@ -534,15 +658,17 @@ cudaError_t launch_pdl(K kern, int grid, int threads, const RankParams& p, cudaS
 
 template <int SC>
 cudaError_t launch_encode(const RankParams& p, cudaStream_t stream) {
+  // the split-row kernel for 4, 8 and 16 stages, the row-per-thread one otherwise
+  constexpr bool kSplit = SC == 4 || SC == 8 || SC == 16;
+  auto kern = kSplit ? rank_encode_split_kernel<kSplit ? SC : 8> : rank_encode_kernel<SC>;
   static int per_sm = 0;  // resident CTAs per SM (same on every GB300)
   if (per_sm == 0 &&
-      (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rank_encode_kernel<SC>, kEncThreads, 0) != cudaSuccess ||
-       per_sm < 1)) {
+      (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kEncThreads, 0) != cudaSuccess || per_sm < 1)) {
     cudaGetLastError();
     per_sm = 1;
   }
   const int grid = static_cast<int>(std::min<int64_t>(p.Tc * p.nblk, int64_t(per_sm) * sm_count()));
-  return launch_pdl(rank_encode_kernel<SC>, grid, kEncThreads, p, stream);
+  return launch_pdl(kern, grid, kEncThreads, p, stream);
 }
 
 }  // namespace
@@ -612,7 +738,7 @@ cudaError_t launch_rank_select(const int64_t* d, int64_t T, int64_t R, int64_t S
       default: e = launch_encode<0>(p, stream); break;
     }
     if (e != cudaSuccess) return e;
-    const int sel_grid = static_cast<int>(std::min<int64_t>(p.Tc * S, int64_t(sms) * 6));
+    const int sel_grid = static_cast<int>(std::min<int64_t>(p.Tc * S, int64_t(sms) * 12));
     count_launch();
     if ((e = launch_pdl(rank_select_kernel, sel_grid, kSelThreads, p, stream)) != cudaSuccess) return e;
   }
