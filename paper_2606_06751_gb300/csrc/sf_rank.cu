@@ -7,9 +7,9 @@
 // kernels run, the encode of the next chunk overlapping the select of this
 // one (programmatic dependent launch, two scratch buffers):
 //  rank_encode_kernel - streams the chunk's rank rows once from HBM (16-byte
-//    loads, two rows in flight per thread, the stage prefix in registers) and
-//    writes every (step, stage)
-//    column as 32-bit keys: the value minus rank 0's value, sign bit flipped,
+//    streaming loads, so that d does not push the scratch out of L2; a row
+//    split over S/2 lanes for 4, 8 or 16 stages) and writes every (step,
+//    stage) column as 32-bit keys: the value minus rank 0's value, sign bit flipped,
 //    so that unsigned key order is value order.  A persistent grid walks
 //    blocks of 2048 rank rows of one step and writes each block's minimum, maximum
 //    and second largest key per stage and a flag for a value 2^31 or more away
@@ -154,8 +154,8 @@ __global__ void __launch_bounds__(kEncThreads) rank_encode_kernel(const RankPara
         const longlong2* rbp = reinterpret_cast<const longlong2*>(dt + (rb + i + (two ? kEncThreads : 0)) * S);
 #pragma unroll
         for (int h = 0; h < SC / 2; ++h) {
-          const longlong2 x = __ldg(ra + h);
-          const longlong2 y = __ldg(rbp + h);
+          const longlong2 x = __ldcs(ra + h);
+          const longlong2 y = __ldcs(rbp + h);
           a[2 * h] = x.x;
           a[2 * h + 1] = x.y;
           b[2 * h] = y.x;
@@ -171,7 +171,7 @@ __global__ void __launch_bounds__(kEncThreads) rank_encode_kernel(const RankPara
 #pragma unroll
         for (int s = 0; s < kCols; ++s) {
           if (s >= S) break;
-          v[s] = __ldg(row + s);
+          v[s] = __ldcs(row + s);
         }
         encode_row(v, i);
       }
@@ -268,7 +268,7 @@ __global__ void __launch_bounds__(kEncThreads) rank_encode_split_kernel(const Ra
 #pragma unroll
       for (int u = 0; u < kUnroll; ++u) {
         const int r = r0 + u * kRowsPerPass + rsub;
-        v[u] = r < nrows ? __ldg(base + int64_t(r) * L) : make_longlong2(0, 0);
+        v[u] = r < nrows ? __ldcs(base + int64_t(r) * L) : make_longlong2(0, 0);
       }
 #pragma unroll
       for (int u = 0; u < kUnroll; ++u) {
