@@ -81,6 +81,8 @@ def lib():
         L.sfo_rank_lag.argtypes = [_P, _I, _I, _I, _P, _P, _P]
         L.sfo_rank_lag.restype = ctypes.c_int
         L.sfo_raw_spread.argtypes = [_P, _I, _I, _I, _I, _I, _P]
+        L.sfo_rank_lag_windows.argtypes = [_P, _I, _I, _I, _I, _I, _P, _P]
+        L.sfo_rank_lag_windows.restype = ctypes.c_int
         L.sfo_raw_spread.restype = ctypes.c_int
         L.sfo_group_windows.argtypes = [_P, _I, _I, _I, _P, _I, _I, _I, _P, _P]
         L.sfo_group_windows.restype = ctypes.c_int
@@ -316,3 +318,14 @@ def stage_group_sum(X, stage_group, K: int) -> np.ndarray:
     Y = np.empty((nW, K), np.int64)
     _check(lib().sfo_stage_group_sum(_ptr(X), nW, S, _ptr(stage_group), K, _ptr(Y)))
     return Y
+
+
+def rank_lag_windows(d, W: int, t0: int = 0):
+    """Sec. 4 lag evidence summed per window: (LW, GW), each [nW][S]."""
+    d = _d(d)
+    T, R, S = d.shape
+    nW = num_windows(t0, T, W)
+    LW = np.empty((nW, S), np.int64)
+    GW = np.empty((nW, S), np.int64)
+    _check(lib().sfo_rank_lag_windows(_ptr(d), T, R, S, t0, W, _ptr(LW), _ptr(GW)))
+    return LW, GW

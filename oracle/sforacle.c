@@ -549,3 +549,24 @@ int sfo_stage_group_sum(const int64_t* X, int64_t nW, int64_t S, const int32_t* 
     for (int64_t s = 0; s < S; ++s) Y[w * K + stage_group[s]] += X[w * S + s];
   return SFO_OK;
 }
+
+int sfo_rank_lag_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W, int64_t* LW,
+                         int64_t* GW) {
+  if (!d || !check_shape(T, R, S) || W < 1 || W > 65536 || t0 < 0) return SFO_BADARG;
+  const int64_t w_first = t0 / W, nW = (t0 + T - 1) / W - w_first + 1;
+  int64_t* L = (int64_t*)malloc(sizeof(int64_t) * (size_t)(T * S));
+  int64_t* G = (int64_t*)malloc(sizeof(int64_t) * (size_t)(T * S));
+  int rc = (L && G) ? sfo_rank_lag(d, T, R, S, L, NULL, G) : SFO_BADARG;
+  if (LW) memset(LW, 0, sizeof(int64_t) * (size_t)(nW * S));
+  if (GW) memset(GW, 0, sizeof(int64_t) * (size_t)(nW * S));
+  for (int64_t t = 0; t < T && rc == SFO_OK; ++t) {
+    const int64_t w = (t0 + t) / W - w_first;
+    for (int64_t s = 0; s < S; ++s) {
+      if (LW) LW[w * S + s] += L[t * S + s]; /* sum_t L[t,s] */
+      if (GW) GW[w * S + s] += G[t * S + s]; /* sum_t G[t,s] */
+    }
+  }
+  free(L);
+  free(G);
+  return rc;
+}

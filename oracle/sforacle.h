@@ -106,6 +106,13 @@ int sfo_rank_lag(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t* L, 
    sum_t (max_r d[t,r,s] - median_r d[t,r,s]), lower median over ranks. */
 int sfo_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W, int64_t* SPREAD);
 
+/* The lag evidence of Sec. 4 per window (windows as in sfo_windows):
+   LW [nW][S] = sum over the window's steps of L[t,s], GW [nW][S] = sum of
+   G[t,s] (the window's delta-lag sums are LW[w][s] - LW[w][s-1]).  Outputs
+   overwritten; each nullable. */
+int sfo_rank_lag_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W, int64_t* LW,
+                         int64_t* GW);
+
 void sfo_config_default(sfo_config* cfg);
 
 /* Frontier within role groups (App. A role check: no global frontier across

@@ -560,3 +560,23 @@ def test_stage_group_sum():
     fb = np.array([0, 1] * 4)                                              # f1 b1 f2 b2 ... -> fwd, bwd
     y = O.stage_group_sum(w.X, fb, 2)
     assert (y[:, 0] == w.X[:, 0::2].sum(axis=1)).all() and (y.sum(axis=1) == w.D).all()
+
+
+def test_lag_windows():
+    # window sums of the per-step evidence; a stall Delta on one of otherwise
+    # identical ranks at step t contributes Delta to every stage from the
+    # stalled one on, in the window of t only
+    rng = np.random.default_rng(21)
+    base = rng.integers(1, 1000, size=(7, 1, 4)).astype(np.int64)
+    d = np.repeat(base, 5, axis=1)
+    d[4, 3, 2] += 555
+    LW, GW = O.rank_lag_windows(d, 3, t0=1)          # windows: steps {0,1}, {2,3,4}, {5,6}
+    assert LW.shape == (3, 4)
+    assert (LW[0] == 0).all() and (LW[2] == 0).all() and list(LW[1]) == [0, 0, 555, 555]
+    assert (GW == LW).all()
+    d2 = rand_d(rng, 20, 6, 3, hi=40, zero_frac=0.2)
+    g = O.rank_lag(d2)
+    LW2, GW2 = O.rank_lag_windows(d2, 7)
+    for w in range(LW2.shape[0]):
+        assert (LW2[w] == g.L[w * 7:(w + 1) * 7].sum(axis=0)).all()
+        assert (GW2[w] == g.G[w * 7:(w + 1) * 7].sum(axis=0)).all()
