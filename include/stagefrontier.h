@@ -162,7 +162,18 @@ sf_status sf_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64
                         int64_t* spread, int32_t accumulate, void* workspace, size_t workspace_bytes,
                         uint32_t* status, cudaStream_t stream);
 
-/* Suggested workspace bytes for sf_rank_lag / sf_raw_spread (0 for a bad shape). */
+/*
+ * sf_rank_lag_windows - the same evidence as window evidence: per window and
+ * stage, Lw = sum_t L[t,s] and Gw = sum_t G[t,s] (the window's delta-lag sums
+ * are Lw[w][s] - Lw[w][s-1]).  Lw, Gw [nW][S] device, nullable (at least
+ * one); windows, t0 and accumulate as in sf_window_aggregate; workspace as in
+ * sf_rank_lag.
+ */
+sf_status sf_rank_lag_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W,
+                              int64_t* Lw, int64_t* Gw, int32_t accumulate, void* workspace, size_t workspace_bytes,
+                              uint32_t* status, cudaStream_t stream);
+
+/* Suggested workspace bytes for sf_rank_lag, sf_rank_lag_windows and sf_raw_spread (0 for a bad shape). */
 size_t sf_rank_workspace_size(int64_t T, int64_t R, int64_t S);
 
 /*

@@ -208,7 +208,8 @@ sf_status sf_rank_lag(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t
     return SF_EINVAL_ALIGN;
   if (!workspace || !rank_workspace_ok(T, R, S, workspace_bytes)) return SF_EWORKSPACE;
   return cuda_status(
-      launch_rank_select(d, T, R, S, 1, 0, 1, L, dL, G, nullptr, workspace, workspace_bytes, status, stream));
+      launch_rank_select(d, T, R, S, 1, 0, 1, L, dL, G, nullptr, nullptr, nullptr, workspace, workspace_bytes,
+                         status, stream));
 }
 
 sf_status sf_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W, int64_t* spread,
@@ -222,7 +223,24 @@ sf_status sf_raw_spread(const int64_t* d, int64_t T, int64_t R, int64_t S, int64
   if (!workspace || !rank_workspace_ok(T, R, S, workspace_bytes)) return SF_EWORKSPACE;
   if (!accumulate && launch_zero(spread, size_t(sf_num_windows(t0, T, W)) * S * 8, stream) != cudaSuccess)
     return SF_ECUDA;
-  return cuda_status(launch_rank_select(d, T, R, S, 0, t0, W, nullptr, nullptr, nullptr, spread, workspace,
+  return cuda_status(launch_rank_select(d, T, R, S, 0, t0, W, nullptr, nullptr, nullptr, nullptr, nullptr, spread,
+                                        workspace, workspace_bytes, status, stream));
+}
+
+sf_status sf_rank_lag_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W,
+                              int64_t* Lw, int64_t* Gw, int32_t accumulate, void* workspace, size_t workspace_bytes,
+                              uint32_t* status, cudaStream_t stream) {
+  if (!d || (!Lw && !Gw) || !shape_ok(T, R, S) || t0 < 0 || W < 1 || W > 65536 ||
+      (accumulate != 0 && accumulate != 1) || t0 > (int64_t(1) << 62) - T)
+    return SF_EINVAL;
+  if (!aligned(d, 16) || !aligned(Lw, 8) || !aligned(Gw, 8) || !aligned(status, 4) || !aligned(workspace, 256))
+    return SF_EINVAL_ALIGN;
+  if (!workspace || !rank_workspace_ok(T, R, S, workspace_bytes)) return SF_EWORKSPACE;
+  const size_t bytes = size_t(sf_num_windows(t0, T, W)) * S * 8;
+  if (!accumulate && ((Lw && launch_zero(Lw, bytes, stream) != cudaSuccess) ||
+                      (Gw && launch_zero(Gw, bytes, stream) != cudaSuccess)))
+    return SF_ECUDA;
+  return cuda_status(launch_rank_select(d, T, R, S, 1, t0, W, nullptr, nullptr, nullptr, Lw, Gw, nullptr, workspace,
                                         workspace_bytes, status, stream));
 }
 

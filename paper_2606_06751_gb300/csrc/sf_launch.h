@@ -58,8 +58,9 @@ cudaError_t launch_stream_pass(const StreamJob& job, cudaStream_t stream);
 cudaError_t launch_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W,
                                  int64_t* m, uint32_t* status, cudaStream_t stream);
 cudaError_t launch_rank_select(const int64_t* d, int64_t T, int64_t R, int64_t S, int of_prefix, int64_t t0,
-                               int64_t W, int64_t* L, int64_t* dL, int64_t* G, int64_t* spread, void* workspace,
-                               size_t ws_bytes, uint32_t* status, cudaStream_t stream);
+                               int64_t W, int64_t* L, int64_t* dL, int64_t* G, int64_t* Lw, int64_t* Gw,
+                               int64_t* spread, void* workspace, size_t ws_bytes, uint32_t* status,
+                               cudaStream_t stream);
 size_t rank_workspace_size(int64_t T, int64_t R, int64_t S);
 bool rank_workspace_ok(int64_t T, int64_t R, int64_t S, size_t bytes);
 cudaError_t launch_group_windows(const int64_t* d, int64_t T, int64_t R, int64_t S, const int32_t* group, int64_t G,

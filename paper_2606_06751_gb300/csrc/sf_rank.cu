@@ -45,8 +45,9 @@ struct RankParams {
   int64_t T, R, S;
   int of_prefix;  // 1: order statistics of P (lag); 0: of d (spread)
   int64_t t0, W, w_first;
-  int64_t *L, *G;   // [T][S], nullable
-  int64_t* spread;  // [nW][S], nullable
+  int64_t *L, *G;    // [T][S], nullable
+  int64_t *Lw, *Gw;  // [nW][S] window sums of L and G, nullable
+  int64_t* spread;   // [nW][S], nullable
   uint32_t* status;
   // one chunk of steps [c0, c0 + Tc) and its scratch
   int64_t c0, Tc;
@@ -576,8 +577,14 @@ __global__ void __launch_bounds__(kSelThreads, 12) rank_select_kernel(const Rank
     if (tid == 0) {
       const int64_t lag = sh.F - sh.med;
       if (p.of_prefix) {
+        const int64_t gap = sh.F - sh.sec;
         if (p.L) p.L[t * S + s] = lag;
-        if (p.G) p.G[t * S + s] = sh.F - sh.sec;
+        if (p.G) p.G[t * S + s] = gap;
+        const int64_t w = (p.t0 + t) / p.W - p.w_first;
+        if (p.Lw && lag)
+          atomicAdd(reinterpret_cast<unsigned long long*>(&p.Lw[w * S + s]), static_cast<unsigned long long>(lag));
+        if (p.Gw && gap)
+          atomicAdd(reinterpret_cast<unsigned long long*>(&p.Gw[w * S + s]), static_cast<unsigned long long>(gap));
       } else {
         const int64_t w = (p.t0 + t) / p.W - p.w_first;
         if (lag) atomicAdd(reinterpret_cast<unsigned long long*>(&p.spread[w * S + s]),
@@ -687,8 +694,9 @@ bool rank_workspace_ok(int64_t T, int64_t R, int64_t S, size_t bytes) {
 }
 
 cudaError_t launch_rank_select(const int64_t* d, int64_t T, int64_t R, int64_t S, int of_prefix, int64_t t0,
-                               int64_t W, int64_t* L, int64_t* dL, int64_t* G, int64_t* spread, void* workspace,
-                               size_t ws_bytes, uint32_t* status, cudaStream_t stream) {
+                               int64_t W, int64_t* L, int64_t* dL, int64_t* G, int64_t* Lw, int64_t* Gw,
+                               int64_t* spread, void* workspace, size_t ws_bytes, uint32_t* status,
+                               cudaStream_t stream) {
   const size_t half = ws_bytes / 2 & ~size_t(255);  // one chunk buffer, 256-byte aligned
   const int64_t Tc = chunk_steps_for(T, R, S, half);
   if (Tc < 1) return cudaErrorInvalidValue;
@@ -706,6 +714,8 @@ cudaError_t launch_rank_select(const int64_t* d, int64_t T, int64_t R, int64_t S
   p.w_first = t0 / W;
   p.L = L ? L : dL;  // without L, the lag is written into dL and converted there
   p.G = G;
+  p.Lw = Lw;
+  p.Gw = Gw;
   p.spread = spread;
   p.status = status;
   p.ldR = l.ldR;

@@ -55,6 +55,7 @@ def _load():
         "sf_topk_suspects": [P, P, I, I, I, I32, P, P, P, P, S],
         "sf_window_baselines": [P, I, I, I, I, I, P, P, P, P, I32, P, S],
         "sf_rank_lag": [P, I, I, I, P, P, P, P, ctypes.c_size_t, P, S],
+        "sf_rank_lag_windows": [P, I, I, I, I, I, P, P, I32, P, ctypes.c_size_t, P, S],
         "sf_group_aggregate": [P, I, I, I, P, I, I, I, P, P, I32, P, S],
         "sf_stage_group_sum": [P, I, I, P, I, P, S],
         "sf_raw_spread": [P, I, I, I, I, I, P, I32, P, ctypes.c_size_t, P, S],
@@ -527,3 +528,19 @@ def sf_gathered_to_steps(src: torch.Tensor, T: int, R: int, S: int, N: int, dst=
     dst = dst if dst is not None else torch.empty((T, R, S), dtype=torch.int64, device=src.device)
     _check(_lib.sf_gathered_to_steps(_p(src), T, R, S, N, _p(dst), _stream(stream)), "sf_gathered_to_steps")
     return dst
+
+
+def sf_rank_lag_windows(d, W: int, t0: int = 0, Lw=None, Gw=None, accumulate: bool = False, workspace=None,
+                        status=None, stream=None):
+    """Window sums of the lag and the gap: (Lw, Gw), each [nW][S]."""
+    T, R, S = _d3(d)
+    nW = num_windows(t0, T, W)
+    Lw = Lw if Lw is not None else _empty((nW, S), torch.int64, d)
+    Gw = Gw if Gw is not None else _empty((nW, S), torch.int64, d)
+    ws = workspace
+    if ws is None:
+        ws = rank_workspace(T, R, S, d.device)
+        _hold([ws], stream)
+    _check(_lib.sf_rank_lag_windows(_p(d), T, R, S, t0, W, _p(Lw), _p(Gw), 1 if accumulate else 0, _p(ws),
+                                    ws.numel(), _p(status), _stream(stream)), "sf_rank_lag_windows")
+    return Lw, Gw

@@ -107,6 +107,9 @@ def test_host_validation(sf):
     assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, None, 0, FAKE, 1 << 20, None, None) == sf.SF_EINVAL
     assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, FAKE, 3, FAKE, 1 << 20, None, None) == sf.SF_EINVAL
     assert L.sf_raw_spread(FAKE, 10, 4, 4, 0, 5, FAKE + 4, 0, FAKE, 1 << 20, None, None) == sf.SF_EINVAL_ALIGN
+    assert L.sf_rank_lag_windows(FAKE, 10, 4, 4, 0, 5, None, None, 0, FAKE, 1 << 20, None, None) == sf.SF_EINVAL
+    assert L.sf_rank_lag_windows(FAKE, 10, 4, 4, 0, 0, FAKE, None, 0, FAKE, 1 << 20, None, None) == sf.SF_EINVAL
+    assert L.sf_rank_lag_windows(FAKE, 10, 4, 4, 0, 5, FAKE, None, 0, FAKE, 8, None, None) == sf.SF_EWORKSPACE
     assert L.sf_rank_workspace_size(8192, 8192, 8) >= 8 * 8192 * 4
     assert L.sf_rank_workspace_size(0, 8, 8) == 0
     # role groups: group count, G*S limit, stage-group ids (host array)

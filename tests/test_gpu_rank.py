@@ -163,3 +163,15 @@ def test_rank_lag_on_workloads(sf, name):
     assert np.array_equal(host(g.L), o.L) and np.array_equal(host(g.dL), o.dL)
     assert np.array_equal(host(g.G), o.G)
     assert np.array_equal(host(sp), O.raw_spread(d_np, w.W))
+
+
+@pytest.mark.parametrize("T,R,S,t0,W", [(37, 3, 5, 0, 7), (300, 64, 8, 5, 100), (45, 1024, 10, 0, 20),
+                                        (9, 8192, 8, 3, 4), (20, 1, 1, 0, 3)])
+def test_rank_lag_windows_parity(sf, T, R, S, t0, W):
+    d_np = make(T, R, S, T * R + S, "lognormal" if R > 3 else "ties")
+    oL, oG = O.rank_lag_windows(d_np, W, t0)
+    st = sf.new_status("cuda")
+    Lw, Gw = sf.sf_rank_lag_windows(dev(d_np), W, t0=t0, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert np.array_equal(host(Lw), oL) and np.array_equal(host(Gw), oG)
