@@ -6,22 +6,23 @@
 // The steps are processed in chunks whose scratch stays in L2; per chunk two
 // kernels run, the encode of the next chunk overlapping the select of this
 // one (programmatic dependent launch, two scratch buffers):
-//  rank_encode_kernel - streams the chunk's rank rows once from HBM (16-byte
-//    streaming loads, so that d does not push the scratch out of L2; a row
-//    split over S/2 lanes for 4, 8 or 16 stages) and writes every (step,
-//    stage) column as 32-bit keys: the value minus rank 0's value, sign bit flipped,
-//    so that unsigned key order is value order.  A persistent grid walks
-//    blocks of 2048 rank rows of one step and writes each block's minimum, maximum
-//    and second largest key per stage and a flag for a value 2^31 or more away
-//    from rank 0's (that step then takes the 64-bit path).
+//  encode (rank_encode_split_kernel for 4, 8 or 16 stages, a rank row split
+//    over S/2 lanes; rank_encode_kernel, a row per thread, otherwise) -
+//    streams the chunk's rank rows once from HBM with streaming loads, so
+//    that d does not push the scratch out of L2, and writes every (step,
+//    stage) column as 32-bit keys: the value minus rank 0's value, sign bit
+//    flipped, so that unsigned key order is value order.  A persistent grid
+//    walks blocks of 2048 rank rows of one step and writes each block's
+//    minimum, maximum and second largest key per stage and a flag for a value
+//    2^31 or more away from rank 0's (that step then takes the 64-bit path).
 //  rank_select_kernel - one CTA per (step, stage) column at a time: radix
 //    selection on the key offsets from the column minimum, the first digit
 //    starting at the highest bit of the range so that it spreads over the 256
 //    bins.  The first pass reads the column from L2 four keys at a time; the
 //    second reads it again, counts the keys in the chosen bin and keeps them
-//    as candidates, so later passes read only those.  Once a column has been read for the
-//    last time its L2 lines are discarded, so the dead scratch is never
-//    written back to HBM.
+//    as candidates, so later passes read only those.  Once a column has been
+//    read for the last time its L2 lines are discarded, so the dead scratch
+//    is never written back to HBM.
 // A last small kernel forms delta-lag from the lag.
 #include <algorithm>
 #include <cstdint>
