@@ -12,7 +12,7 @@
 //    that d does not push the scratch out of L2, and writes every (step,
 //    stage) column as 32-bit keys: the value minus rank 0's value, sign bit
 //    flipped, so that unsigned key order is value order.  A persistent grid
-//    walks blocks of 2048 rank rows of one step and writes each block's
+//    walks blocks of 1024 rank rows of one step and writes each block's
 //    minimum, maximum and second largest key per stage and a flag for a value
 //    2^31 or more away from rank 0's (that step then takes the 64-bit path).
 //  rank_select_kernel - one CTA per (step, stage) column at a time: radix
@@ -35,7 +35,7 @@ namespace {
 
 constexpr int kRkMaxS = 32;
 constexpr int kEncThreads = 256;
-constexpr int kEncRows = 2048;  // rank rows per encode item (8 per thread)
+constexpr int kEncRows = 1024;  // rank rows per encode item (4 per thread)
 constexpr int kSelThreads = 128;
 constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kSelCand = 2048;  // candidate keys a column may keep after the second pass
