@@ -145,8 +145,10 @@ __device__ __forceinline__ uint32_t warp_select_bits32(const uint32_t (&x)[NPL],
   if (hi == 0) return prefix;
   uint32_t* ncand = hist + 256;  // spare word after the bins
   if (kept <= 32) {
-    // at most one value of the chosen bin per lane: gather them and take the
-    // rem-th smallest by counting, instead of more histogram passes
+    // at most one value of the chosen bin per lane: gather them, sort the
+    // warp's 32 values with a bitonic network (lanes past the bin hold the
+    // largest key, which sorts last) and take the rem-th smallest, instead
+    // of more histogram passes
     __syncwarp();
     if (lane == 0) *ncand = 0;
     __syncwarp();
@@ -154,18 +156,18 @@ __device__ __forceinline__ uint32_t warp_select_bits32(const uint32_t (&x)[NPL],
     for (int i = 0; i < NPL; ++i)
       if ((x[i] >> hi) == digit) *cand(atomicAdd(ncand, 1u)) = x[i];
     __syncwarp();
-    const bool mine = static_cast<uint32_t>(lane) < kept;
-    const uint32_t v = mine ? *cand(lane) : 0u;
-    uint32_t lt = 0, le = 0;
+    uint32_t v = static_cast<uint32_t>(lane) < kept ? *cand(lane) : 0xffffffffu;
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
-      const uint32_t c = __shfl_sync(kFull, v, j);
-      const bool live = static_cast<uint32_t>(j) < kept;
-      lt += (live && c < v) ? 1u : 0u;
-      le += (live && c <= v) ? 1u : 0u;
+    for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+      for (int stride = size >> 1; stride > 0; stride >>= 1) {
+        const uint32_t o = __shfl_xor_sync(kFull, v, stride);
+        // ascending within blocks whose `size` bit is clear; the lower lane of a pair keeps the smaller
+        const bool up = (lane & size) == 0, low = (lane & stride) == 0;
+        v = (up == low) ? min(v, o) : max(v, o);
+      }
     }
-    const uint32_t hit = __ballot_sync(kFull, mine && lt <= rem && rem < le);
-    const uint32_t ans = __shfl_sync(kFull, v, __ffs(hit) - 1);
+    const uint32_t ans = __shfl_sync(kFull, v, static_cast<int>(rem));
     __syncwarp();
     return ans;
   }
