@@ -149,7 +149,8 @@ def test_topk_parity(sf, nW, S, R, k):
     assert np.array_equal(host(t.pair), o.pair) and np.array_equal(host(t.pair_value), o.pair_value)
 
 
-@pytest.mark.parametrize("T,R,S,W", [(100, 8, 6, 100), (250, 4, 3, 32), (130, 5, 4, 64), (300, 2, 8, 128),
+@pytest.mark.parametrize("T,R,S,W", [(7, 3, 5, 1), (9, 4, 3, 2), (33, 2, 3, 3),
+                                     (100, 8, 6, 100), (250, 4, 3, 32), (130, 5, 4, 64), (300, 2, 8, 128),
                                      (700, 3, 2, 256), (1100, 2, 4, 512), (2100, 1, 4, 1000),
                                      (2200, 2, 2, 1024), (2500, 1, 3, 1100), (45, 1024, 10, 20)])
 @pytest.mark.parametrize("kind", ["ties", "lognormal", "wide", "zeros", "ranges", "clusters"])
@@ -172,7 +173,8 @@ def test_median_parity(sf, T, R, S, W, kind):
 
 
 @pytest.mark.parametrize("T,R,S,W", [(120, 8, 6, 50), (64, 128, 8, 30), (40, 1024, 10, 16),
-                                     (33, 3, 5, 10), (20, 8192, 8, 8), (30, 64, 16, 30)])
+                                     (33, 3, 5, 10), (20, 8192, 8, 8), (30, 64, 16, 30), (9, 5, 4, 1),
+                                     (11, 40, 8, 2)])
 def test_direct_gain_parity(sf, T, R, S, W):
     d_np = make(T, R, S, R + S, "lognormal")
     m_np = O.window_median(d_np, W)
