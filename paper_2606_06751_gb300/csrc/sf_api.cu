@@ -1,7 +1,8 @@
 // sf_api.cu - the C ABI of libstagefrontier (declared in stagefrontier.h):
 // argument validation, output clearing, workspace carving and launch
-// sequencing.  Every computation happens in the kernels of sf_stream.cu and
-// sf_select.cu; this file performs no arithmetic on the data.
+// sequencing.  Every computation happens in the kernels (sf_stream.cu,
+// sf_select.cu, sf_rank.cu, sf_group.cu, sf_ingest.cu); this file performs no
+// arithmetic on the data.
 #include <atomic>
 #include <cstring>
 
