@@ -514,6 +514,61 @@ def run_reference(args):
     }
 
 
+def run_configs(args):
+    """Throughput of the frontier pass (sf_frontier), the aggregation pass
+    (sf_window_aggregate) and the whole step on every synthetic configuration:
+    the four workloads and the 1 GiB bandwidth sweep.  One GPU; one JSON line
+    with a record per configuration."""
+    device = torch.device("cuda", 0)
+    torch.cuda.set_device(device)
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_06751_gb300 import stagefrontier as sf
+
+    peak, peak_kind = peaks()
+    names = ["tiny", "ddp128", "fsdp1024", "accum8192"] + [f"sweep_R{R}_S{S}" for R in wl.SWEEP_R
+                                                           for S in wl.SWEEP_S]
+    if args.only:
+        names = [n for n in names if n in args.only.split(",")]
+    out = []
+    for name in names:
+        if name.startswith("sweep_"):
+            R, S = (int(x[1:]) for x in name.split("_")[1:])
+            w = wl.sweep(R, S, seed=args.seed)
+        else:
+            w = wl.by_name(name, seed=args.seed)
+        host = torch.empty((w.T, w.R, w.S), dtype=torch.int64, pin_memory=True)
+        w.fill(host.numpy().reshape(-1), threads=os.cpu_count() or 1)
+        d = host.to(device)
+        del host
+        st = sf.new_status(device)
+        nW = sf.num_windows(0, w.T, w.W)
+        e = lambda shape, dt: torch.empty(shape, dtype=dt, device=device)  # noqa: E731
+        fr = (e((w.T, w.S), torch.int64), e((w.T, w.S), torch.int32), e((w.T,), torch.int64))
+        frontier = lambda: sf.sf_frontier(d, a=fr[0], lead=fr[1], makespan=fr[2], status=st)  # noqa: E731
+        pipe = Pipeline(sf, w, d)
+        din = w.T * w.R * w.S * 8
+        rec = {"config": name, "R": w.R, "S": w.S, "T": w.T, "W": w.W, "gbytes": round(din / 1e9, 3)}
+        f_secs = timed_loop(frontier, args.steps, args.warmup, 1, device, True) / args.steps
+        f_bytes = din + w.T * w.S * 12 + w.T * 8
+        rec["frontier"] = {"ms": round(f_secs * 1e3, 4), "gbs": round(f_bytes / f_secs / 1e9, 1),
+                           "frac": round(f_bytes / f_secs / 1e9 / peak, 4), "records_per_s": w.records / f_secs}
+        a_secs = timed_loop(pipe.aggregate, args.steps, args.warmup, 1, device, True) / args.steps
+        a_bytes = pipe.algorithmic_bytes()["window_aggregate"]
+        rec["aggregate"] = {"ms": round(a_secs * 1e3, 4), "gbs": round(a_bytes / a_secs / 1e9, 1),
+                            "frac": round(a_bytes / a_secs / 1e9 / peak, 4)}
+        s_secs = timed_loop(pipe.step, args.steps, args.warmup, 1, device, True) / args.steps
+        rec["step"] = {"ms": round(s_secs * 1e3, 4), "records_per_s": w.records / s_secs}
+        torch.cuda.synchronize()
+        rec["status"] = int(st.item()) | int(pipe.status.item())
+        out.append(rec)
+        del d, pipe, fr
+        torch.cuda.empty_cache()
+    return {"metric": "per-configuration throughput (frontier pass, aggregation pass, whole step)",
+            "unit": "GB/s and records/s", "peak_gbs": peak, "peak_kind": peak_kind, "steps": args.steps,
+            "warmup": args.warmup, "configs": out}
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -526,10 +581,16 @@ def main(argv=None):
     ap.add_argument("--cpu-sample-windows", type=int, default=2)
     ap.add_argument("--ref-sample-steps", type=int, default=100)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--configs", action="store_true",
+                    help="throughput on every synthetic configuration instead of the benchmark step")
+    ap.add_argument("--only", default=None, help="with --configs: comma-separated configuration names")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
-    line = run_reference(args) if args.impl == "reference" else run_ours(args)
+    if args.configs:
+        line = run_configs(args)
+    else:
+        line = run_reference(args) if args.impl == "reference" else run_ours(args)
     if line is not None:
         print(json.dumps(line), flush=True)
     if torch.distributed.is_initialized():
