@@ -489,16 +489,16 @@ __global__ void __launch_bounds__(kSelThreads, 12) rank_select_kernel(const Rank
       if (nb > 0) {
         for (int i = tid; i < 256; i += kSelThreads) sh.hist[i] = 0;
         __syncthreads();
-        const int shift = nb > 8 ? nb - 8 : 0;  // offsets are below 2^nb: no mask needed
+        const int shift = nb > 8 ? nb - 8 : 0;  // offsets are below 2^nb; the mask only guards the bins
         const int nq = R >> 2;
         for (int i = tid; i < nq; i += kSelThreads) {
           const uint4 k4 = reinterpret_cast<const uint4*>(col)[i];
-          atomicAdd(&sh.hist[(k4.x - lo) >> shift], 1u);
-          atomicAdd(&sh.hist[(k4.y - lo) >> shift], 1u);
-          atomicAdd(&sh.hist[(k4.z - lo) >> shift], 1u);
-          atomicAdd(&sh.hist[(k4.w - lo) >> shift], 1u);
+          atomicAdd(&sh.hist[((k4.x - lo) >> shift) & 255u], 1u);
+          atomicAdd(&sh.hist[((k4.y - lo) >> shift) & 255u], 1u);
+          atomicAdd(&sh.hist[((k4.z - lo) >> shift) & 255u], 1u);
+          atomicAdd(&sh.hist[((k4.w - lo) >> shift) & 255u], 1u);
         }
-        for (int r = 4 * nq + tid; r < R; r += kSelThreads) atomicAdd(&sh.hist[(col[r] - lo) >> shift], 1u);
+        for (int r = 4 * nq + tid; r < R; r += kSelThreads) atomicAdd(&sh.hist[((col[r] - lo) >> shift) & 255u], 1u);
         __syncthreads();
         if (warp == 0) {
           uint32_t digit, below;
@@ -651,11 +651,11 @@ int64_t chunk_steps_for(int64_t T, int64_t R, int64_t S, size_t bytes) {
 }
 
 template <typename K>
-cudaError_t launch_pdl(K kern, int grid, int threads, const RankParams& p, cudaStream_t stream) {
+cudaError_t launch_pdl(K kern, int grid, int threads, const RankParams& p, cudaStream_t stream, bool overlap = true) {
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[0].val.programmaticStreamSerializationAllowed = overlap ? 1 : 0;
   cfg.gridDim = dim3(static_cast<unsigned>(grid));
   cfg.blockDim = dim3(static_cast<unsigned>(threads));
   cfg.stream = stream;
@@ -664,8 +664,11 @@ cudaError_t launch_pdl(K kern, int grid, int threads, const RankParams& p, cudaS
   return cudaLaunchKernelEx(&cfg, kern, p);
 }
 
+// first: the call's first chunk.  Its encode starts only once everything
+// before it on the stream has completed: the previous call's last select may
+// still be reading the same scratch buffer.
 template <int SC>
-cudaError_t launch_encode(const RankParams& p, cudaStream_t stream) {
+cudaError_t launch_encode(const RankParams& p, cudaStream_t stream, bool first) {
   // the split-row kernel for 4, 8 and 16 stages, the row-per-thread one otherwise
   constexpr bool kSplit = SC == 4 || SC == 8 || SC == 16;
   auto kern = kSplit ? rank_encode_split_kernel<kSplit ? SC : 8> : rank_encode_kernel<SC>;
@@ -676,7 +679,7 @@ cudaError_t launch_encode(const RankParams& p, cudaStream_t stream) {
     per_sm = 1;
   }
   const int grid = static_cast<int>(std::min<int64_t>(p.Tc * p.nblk, int64_t(per_sm) * sm_count()));
-  return launch_pdl(kern, grid, kEncThreads, p, stream);
+  return launch_pdl(kern, grid, kEncThreads, p, stream, !first);
 }
 
 }  // namespace
@@ -741,12 +744,12 @@ cudaError_t launch_rank_select(const int64_t* d, int64_t T, int64_t R, int64_t S
     count_launch();
     cudaError_t e;
     switch (S) {
-      case 4: e = launch_encode<4>(p, stream); break;
-      case 6: e = launch_encode<6>(p, stream); break;
-      case 8: e = launch_encode<8>(p, stream); break;
-      case 10: e = launch_encode<10>(p, stream); break;
-      case 16: e = launch_encode<16>(p, stream); break;
-      default: e = launch_encode<0>(p, stream); break;
+      case 4: e = launch_encode<4>(p, stream, c == 0); break;
+      case 6: e = launch_encode<6>(p, stream, c == 0); break;
+      case 8: e = launch_encode<8>(p, stream, c == 0); break;
+      case 10: e = launch_encode<10>(p, stream, c == 0); break;
+      case 16: e = launch_encode<16>(p, stream, c == 0); break;
+      default: e = launch_encode<0>(p, stream, c == 0); break;
     }
     if (e != cudaSuccess) return e;
     const int sel_grid = static_cast<int>(std::min<int64_t>(p.Tc * S, int64_t(sms) * 12));

@@ -175,3 +175,27 @@ def test_rank_lag_windows_parity(sf, T, R, S, t0, W):
     torch.cuda.synchronize()
     assert int(st.item()) == 0
     assert np.array_equal(host(Lw), oL) and np.array_equal(host(Gw), oG)
+
+
+def test_back_to_back_calls_share_the_workspace(sf):
+    """Calls queued back to back on one stream reuse one workspace: a call's
+    first chunk must not overwrite the scratch the previous call's last
+    chunk is still selecting from (several chunks per call, odd and even
+    chunk counts)."""
+    T, R, S, W = 700, 2048, 8, 100
+    d_np = make(T, R, S, 77, "lognormal")
+    d = dev(d_np)
+    one = int(sf.lib().sf_rank_workspace_size(1, R, S))
+    o_sp = O.raw_spread(d_np, W)
+    o_lag = O.rank_lag(d_np)
+    for steps_per_chunk in (64, 100, 233):
+        ws = torch.empty(one * steps_per_chunk, dtype=torch.uint8, device="cuda")
+        outs = []
+        for _ in range(4):
+            outs.append(sf.sf_raw_spread(d, W, workspace=ws))
+            outs.append(sf.sf_rank_lag(d, out=sf.Lag(None, None, torch.empty((T, S), dtype=torch.int64,
+                                                                             device="cuda")), workspace=ws).G)
+        torch.cuda.synchronize()
+        for i in range(0, len(outs), 2):
+            assert np.array_equal(host(outs[i]), o_sp), (steps_per_chunk, i)
+            assert np.array_equal(host(outs[i + 1]), o_lag.G), (steps_per_chunk, i)
