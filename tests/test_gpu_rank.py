@@ -52,7 +52,8 @@ def make(T, R, S, seed, kind):
 SHAPES = [(20, 1, 1), (9, 2, 3), (37, 3, 5), (11, 7, 32), (6, 5, 18), (50, 2, 8),
           (1000, 8, 6), (123, 64, 4), (97, 40, 10), (77, 64, 16), (31, 257, 8),
           (13, 1024, 10), (7, 8192, 8), (5, 4096, 16), (3, 32768, 4), (2, 65536, 2), (2, 65535, 7),
-          (2, 32768, 16), (3, 9000, 9), (2, 65536, 32)]
+          (2, 32768, 16), (3, 9000, 9), (2, 65536, 32),
+          (5, 1023, 4), (4, 2048, 5), (3, 2049, 7), (3, 4097, 3), (2, 6001, 12)]
 
 
 @pytest.mark.parametrize("T,R,S", SHAPES)
