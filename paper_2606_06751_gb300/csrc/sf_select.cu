@@ -37,10 +37,10 @@ __global__ void zero_kernel(uint32_t* __restrict__ p, size_t words) {
 constexpr int kMedCols = 8;
 constexpr int kMedThreads = kMedCols * 32;
 constexpr int kMedBins = 256;
-// Per-warp counters: 256 digit bins, then 32 per-lane discard slots that
-// non-matching and padding values increment instead of branching around the
-// atomic.  288 words = 1152 bytes keeps every warp's block 16-byte aligned.
-constexpr int kMedHistWords = kMedBins + 32;
+// Per-warp counters: 256 digit bins, then 48 spare words (a compacted bin of
+// at most 32 values and its padding to whole 16-byte groups).  304 words =
+// 1216 bytes keeps every warp's block 16-byte aligned.
+constexpr int kMedHistWords = kMedBins + 48;
 
 // k-th smallest (0-based) of the lane-strided values get(i) (row lane + 32 i,
 // valid while row < n), all below 2^nbits.  hist: this warp's 256 counters.
@@ -113,104 +113,6 @@ __device__ __forceinline__ void red_shared_inc_if(uint32_t* counter, bool pred) 
       : "memory");
 }
 
-// The k-th smallest of the live values among x[i] (row lane + 32 i), all
-// below 2^nbits.  Padding slots must hold 2^nbits - 1: they sort at or after
-// every live value, so counting them never moves the rank-k bin and no slot
-// needs a validity test.  The first digit takes the top 8 bits of the range,
-// [nbits - 8, nbits), so it spreads over the 256 bins and its chosen bin
-// usually holds a few percent of the column; the next pass then keeps the
-// values of that bin as candidates (in this warp's own, already consumed
-// column slots of the tile: slot j at cand(j)) and every later pass reads only
-// those; a bin of at most 32 values is finished directly, one value per lane,
-// by counting.  A bin too full to keep (heavy ties) falls back to predicated
-// increments over all slots.
-template <int NPL, typename CandAddr>
-__device__ __forceinline__ uint32_t warp_select_bits32(const uint32_t (&x)[NPL], int nbits, uint32_t k,
-                                                       uint32_t* hist, int lane, CandAddr cand) {
-  constexpr uint32_t kCap = 32u * NPL < 512u ? 32u * NPL : 512u;  // candidate slots
-  if (nbits == 0) return 0;
-  int sh = nbits > 8 ? nbits - 8 : 0;
-  reinterpret_cast<uint4*>(hist)[2 * lane] = make_uint4(0, 0, 0, 0);
-  reinterpret_cast<uint4*>(hist)[2 * lane + 1] = make_uint4(0, 0, 0, 0);
-  __syncwarp();
-#pragma unroll
-  for (int i = 0; i < NPL; ++i) atomicAdd(&hist[x[i] >> sh], 1u);  // x < 2^nbits: the bin is below 256
-  __syncwarp();
-  uint32_t digit, below;
-  hist_find(hist, k, lane, digit, below);
-  uint32_t rem = k - below;
-  uint32_t prefix = digit << sh;
-  const uint32_t kept = hist[digit];  // values the next pass matches
-  int hi = sh;                        // offset bits at and above hi are chosen
-  if (hi == 0) return prefix;
-  uint32_t* ncand = hist + 256;  // spare word after the bins
-  if (kept <= 32) {
-    // at most one value of the chosen bin per lane: gather them, sort the
-    // warp's 32 values with a bitonic network (lanes past the bin hold the
-    // largest key, which sorts last) and take the rem-th smallest, instead
-    // of more histogram passes
-    __syncwarp();
-    if (lane == 0) *ncand = 0;
-    __syncwarp();
-#pragma unroll
-    for (int i = 0; i < NPL; ++i)
-      if ((x[i] >> hi) == digit) *cand(atomicAdd(ncand, 1u)) = x[i];
-    __syncwarp();
-    uint32_t v = static_cast<uint32_t>(lane) < kept ? *cand(lane) : 0xffffffffu;
-#pragma unroll
-    for (int size = 2; size <= 32; size <<= 1) {
-#pragma unroll
-      for (int stride = size >> 1; stride > 0; stride >>= 1) {
-        const uint32_t o = __shfl_xor_sync(kFull, v, stride);
-        // ascending within blocks whose `size` bit is clear; the lower lane of a pair keeps the smaller
-        const bool up = (lane & size) == 0, low = (lane & stride) == 0;
-        v = (up == low) ? min(v, o) : max(v, o);
-      }
-    }
-    const uint32_t ans = __shfl_sync(kFull, v, static_cast<int>(rem));
-    __syncwarp();
-    return ans;
-  }
-  const bool compact = kept <= kCap;
-  bool keep_pass = compact;  // the next pass keeps the candidates
-  __syncwarp();
-  while (hi > 0) {
-    sh = hi > 8 ? hi - 8 : 0;
-    const uint32_t mask = (1u << (hi - sh)) - 1u;
-    reinterpret_cast<uint4*>(hist)[2 * lane] = make_uint4(0, 0, 0, 0);
-    reinterpret_cast<uint4*>(hist)[2 * lane + 1] = make_uint4(0, 0, 0, 0);
-    if (lane == 0) *ncand = 0;
-    __syncwarp();
-    if (!compact) {
-#pragma unroll
-      for (int i = 0; i < NPL; ++i)
-        red_shared_inc_if(&hist[(x[i] >> sh) & mask], (x[i] >> hi) == (prefix >> hi));
-    } else if (keep_pass) {
-      // the pass after the first: count and keep the matching values
-#pragma unroll
-      for (int i = 0; i < NPL; ++i) {
-        if ((x[i] >> hi) == (prefix >> hi)) {
-          atomicAdd(&hist[(x[i] >> sh) & mask], 1u);
-          *cand(atomicAdd(ncand, 1u)) = x[i];
-        }
-      }
-    } else {
-      for (uint32_t j = lane; j < kept; j += 32) {
-        const uint32_t v = *cand(j);
-        red_shared_inc_if(&hist[(v >> sh) & mask], (v >> hi) == (prefix >> hi));
-      }
-    }
-    __syncwarp();
-    hist_find(hist, rem, lane, digit, below);
-    rem -= below;
-    prefix |= digit << sh;
-    hi = sh;
-    keep_pass = false;
-    __syncwarp();
-  }
-  return prefix;
-}
-
 template <int NPL, bool kVec>
 __global__ void __launch_bounds__(kMedThreads)
     median_kernel(const int64_t* __restrict__ d, int64_t T, int64_t RS, int64_t W, int64_t ngroups,
@@ -273,123 +175,215 @@ __global__ void __launch_bounds__(kMedThreads)
   if (lane == 0) m[w * RS + c0 + warp] = static_cast<int64_t>((lo + ans) ^ kSign);
 }
 
-// The same selection with the window tile brought in by bulk tensor copies: one
-// thread issues the whole (window x 8 columns) tile, up to four 2-D boxes of
-// 8 int64 x box_rows, all completing on one mbarrier.  The tile stays row-major
-// (64-byte rows) with the 64-byte swizzle, so a warp reading one column down
-// 32 rows touches 8 distinct 16-byte bank groups per 16 lanes.  Offsets from
-// the column minimum stay in registers only when they fit 32 bits; wider
-// columns re-read shared memory on every radix pass.  Registers are capped so
-// three CTAs share an SM and one CTA's copy overlaps another's selection.
+// Radix selection on a column held in registers (x[i] = row lane + 32 i):
+// the k-th smallest of the live values, all below 2^nbits.  Padding slots
+// must hold 2^nbits - 1: they sort at or after every live value, so counting
+// them never moves the rank-k bin and no slot needs a validity test.  The
+// first digit is the top 8 bits of the range, [nbits - 8, nbits), so it
+// spreads over the 256 bins and its chosen bin usually holds a few percent of
+// the column; each later pass counts, predicated, the values that share the
+// digits chosen so far.  As soon as the chosen bin holds at most 32 values
+// they are compacted into the spare words after the bins (ballot ranks, no
+// atomics) and each is ranked by counting.
 template <int NPL>
+__device__ __forceinline__ uint32_t warp_select_regs(const uint32_t (&x)[NPL], int nbits, uint32_t k,
+                                                     uint32_t* hist, int lane) {
+  uint32_t prefix = 0, rem = k;
+  int hi = nbits;
+  bool first = true;
+  while (hi > 0) {
+    const int sh = hi > 8 ? hi - 8 : 0;
+    const uint32_t mask = (1u << (hi - sh)) - 1u;
+    reinterpret_cast<uint4*>(hist)[2 * lane] = make_uint4(0, 0, 0, 0);
+    reinterpret_cast<uint4*>(hist)[2 * lane + 1] = make_uint4(0, 0, 0, 0);
+    __syncwarp();
+    if (first) {
+#pragma unroll
+      for (int i = 0; i < NPL; ++i) atomicAdd(&hist[x[i] >> sh], 1u);  // x < 2^nbits: the bin is below 256
+    } else {
+#pragma unroll
+      for (int i = 0; i < NPL; ++i)
+        red_shared_inc_if(&hist[(x[i] >> sh) & mask], (x[i] >> hi) == (prefix >> hi));
+    }
+    __syncwarp();
+    uint32_t digit, below;
+    hist_find(hist, rem, lane, digit, below);
+    const uint32_t kept = hist[digit];
+    rem -= below;
+    prefix |= digit << sh;
+    hi = sh;
+    first = false;
+    if (hi > 0 && kept <= 32) {
+      uint32_t* cbuf = hist + kMedBins;
+      const uint32_t below_lane = (1u << lane) - 1u;
+      uint32_t base = 0;
+#pragma unroll
+      for (int i = 0; i < NPL; ++i) {
+        const bool mt = (x[i] >> hi) == (prefix >> hi);
+        const uint32_t mm = __ballot_sync(kFull, mt);
+        if (mm) {
+          if (mt) cbuf[base + __popc(mm & below_lane)] = x[i];
+          base += __popc(mm);
+        }
+      }
+      if (lane < 3) cbuf[kept + lane] = 0xffffffffu;  // pad to whole 16-byte groups (kept + 3 <= 35 < 64 spare)
+      __syncwarp();
+      // rank each bin value by counting (broadcast reads of the bin): the
+      // answer is a value with lt <= rem < le.  Padding counts only toward
+      // le of the largest key, which no rank below kept can need.
+      const uint32_t v = cbuf[lane & 31];
+      uint32_t lt = 0, le = 0;
+      for (uint32_t q = 0; q < kept; q += 4) {
+        const uint4 c = *reinterpret_cast<const uint4*>(cbuf + q);
+        lt += (c.x < v) + (c.y < v) + (c.z < v) + (c.w < v);
+        le += (c.x <= v) + (c.y <= v) + (c.z <= v) + (c.w <= v);
+      }
+      const uint32_t hit = __ballot_sync(kFull, static_cast<uint32_t>(lane) < kept && lt <= rem && rem < le);
+      const uint32_t ans = __shfl_sync(kFull, v, __ffs(hit) - 1);
+      __syncwarp();
+      return ans;
+    }
+    __syncwarp();
+  }
+  return prefix;
+}
+
+// Lower median of one column of n <= 32 NPL rows read from global memory
+// (stride RS) on every pass, on 64-bit order-preserving keys: the path of a
+// column whose values do not share their high 32 bits.  Kept out of line so
+// its registers do not weigh on the 32-bit path.
+template <int NPL>
+__device__ __noinline__ int64_t median_column_global(const int64_t* __restrict__ dc, int64_t RS, int n, uint32_t* hist,
+                                                     int lane) {
+  constexpr uint64_t kSign = 1ull << 63;
+  auto ukey = [&](int i) { return static_cast<uint64_t>(__ldg(dc + int64_t(lane + 32 * i) * RS)) ^ kSign; };
+  uint64_t lo = ~0ull, hi = 0;
+#pragma unroll 4
+  for (int i = 0; i < NPL; ++i)
+    if (lane + 32 * i < n) {
+      const uint64_t u = ukey(i);
+      lo = u < lo ? u : lo;
+      hi = u > hi ? u : hi;
+    }
+  lo = warp_min_u64(lo);
+  hi = warp_max_u64(hi);
+  const uint64_t range = hi - lo;
+  const int nbits = range ? 64 - __clzll(static_cast<long long>(range)) : 0;
+  const uint32_t k = static_cast<uint32_t>((n - 1) / 2);
+  const uint64_t key =
+      lo + warp_radix_select<uint64_t, NPL>([&](int i) { return ukey(i) - lo; }, n, nbits, k, hist, lane);
+  return static_cast<int64_t>(key ^ kSign);
+}
+
+// Persistent form of the median: each CTA walks (window, 8-column) tiles
+// with one tile buffer and two mbarriers.  `full` completes when a tile's
+// bulk copies have landed; each warp copies its column into registers and
+// arrives on `empty`, and once all eight have, one thread issues the copies
+// of the CTA's next tile into the same buffer, so the copy runs under the
+// selection of the current tile and no CTA-wide barrier aligns the warps.
+// The selection touches only registers and the warp's counters.  A column
+// whose values do not share their high 32 bits selects on 64-bit values
+// re-read from d.  Every window of a launch holds the same n rows.
+template <int NPL, bool kFit>
 __global__ void __launch_bounds__(kMedThreads, 3)
-    median_tma_kernel(const __grid_constant__ CUtensorMap map, int64_t T, int64_t RS, int64_t W,
-                      int64_t ngroups, int box_rows, int nbox, int tile_rows, int64_t* __restrict__ m,
-                      uint32_t* status) {
+    median_persist_kernel(const __grid_constant__ CUtensorMap map, const int64_t* __restrict__ d, int64_t T,
+                          int64_t RS, int64_t W, int64_t w0, int64_t nW, int64_t ngroups, int box_rows, int nbox,
+                          int64_t* __restrict__ m, uint32_t* status) {
   extern __shared__ unsigned char smem_raw[];
   unsigned char* tile = align_1024(smem_raw);
   const uint32_t tile_bytes = uint32_t(nbox) * uint32_t(box_rows) * 64u;  // bytes the copies write
+  const int tile_rows = max(nbox * box_rows, 32 * NPL);
   uint32_t* hists = reinterpret_cast<uint32_t*>(tile + uint32_t(tile_rows) * 64u);
-  uint64_t* bar = reinterpret_cast<uint64_t*>(hists + kMedCols * kMedHistWords);
-  volatile int* abort = reinterpret_cast<volatile int*>(bar + 1);
-  const int64_t w = blockIdx.x / ngroups;
-  const int64_t c0 = (blockIdx.x % ngroups) * kMedCols;
-  const int ncols = static_cast<int>(imin64(kMedCols, RS - c0));
-  const int64_t tb = w * W;
-  const int n = static_cast<int>(imin64(W, T - tb));
+  uint64_t* full = reinterpret_cast<uint64_t*>(hists + kMedCols * kMedHistWords);
+  uint64_t* empty = full + 1;
+  volatile int* abort = reinterpret_cast<volatile int*>(full + 2);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  uint32_t* hist = hists + warp * kMedHistWords;
+  const int64_t ntiles = nW * ngroups;
+  auto issue = [&](int64_t id) {  // one thread: the bulk copies of tile `id`
+    const int64_t c0 = (id % ngroups) * kMedCols;
+    const int64_t tb = (w0 + id / ngroups) * W;
+    mbar_arrive_expect_tx(full, tile_bytes);
+    for (int b = 0; b < nbox; ++b)
+      tma_load_2d(tile + size_t(b) * box_rows * 64, &map, static_cast<int32_t>(c0),
+                  static_cast<int32_t>(tb + int64_t(b) * box_rows), full);
+  };
   if (threadIdx.x == 0) {
-    mbar_init(bar, 1);
+    mbar_init(full, 1);
+    mbar_init(empty, kMedCols);
     *abort = 0;
     fence_barrier_init();
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    mbar_arrive_expect_tx(bar, tile_bytes);
-    for (int b = 0; b < nbox; ++b)
-      tma_load_2d(tile + size_t(b) * box_rows * 64, &map, static_cast<int32_t>(c0),
-                  static_cast<int32_t>(tb + int64_t(b) * box_rows), bar);
-  }
-  const bool ok = mbar_wait_bounded(bar, 0, abort);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (!ok) {
-    if (threadIdx.x == 0) {
-      report(status, SF_ST_TIMEOUT);
-      mbar_wait_timeout(bar, 0);  // let the copies land before the CTA's memory is released
-    }
-    return;
-  }
-  if (warp >= ncols) return;
-  uint32_t* hist = hists + warp * kMedHistWords;
-  // Row lane + 32 i of this warp's column: the 64-byte swizzle term depends
-  // only on (row >> 1) & 3 = (lane >> 1) & 3, so each lane has one base and a
-  // fixed 2048-byte stride.
-  const unsigned char* col = tile + lane * 64 + ((((warp >> 1) ^ ((lane >> 1) & 3)) << 4) | ((warp & 1) << 3));
-  // Order-preserving unsigned key of a signed value: flip the sign bit, i.e.
-  // bit 31 of the high word.  Most columns share one high word; then the
-  // whole selection runs on the 32-bit low words.
-  uint32_t xl[NPL];
-  const int live = n - lane;  // slot i holds a row of the window iff 32 i < live
-  // Low-word min/max over pairs of slots with 3-input min/max; a padding slot
-  // repeats row 0's value (row 0 is always in the window) so it cannot move
-  // either.  High words only need to agree: OR-accumulate their differences
-  // from row 0's high word.
-  const uint2 own0 = *reinterpret_cast<const uint2*>(col);  // lane 0's first slot is row 0
-  const uint32_t ref_x = __shfl_sync(kFull, own0.x, 0);
-  const uint32_t ref_y = __shfl_sync(kFull, own0.y, 0);
-  uint32_t lmin = ref_x, lmax = ref_x, hdiff = 0;
-#pragma unroll
-  for (int i = 0; i < NPL; ++i) {
-    const uint2 v = *reinterpret_cast<const uint2*>(col + i * 2048);  // in the tile even for padding slots
-    const bool ok = 32 * i < live;
-    xl[i] = ok ? v.x : ref_x;
-    hdiff |= ok ? (v.y ^ ref_y) : 0u;
-  }
-#pragma unroll
-  for (int i = 0; i + 1 < NPL; i += 2) {
-    lmin = __vimin3_u32(lmin, xl[i], xl[i + 1]);
-    lmax = __vimax3_u32(lmax, xl[i], xl[i + 1]);
-  }
-  if (NPL & 1) {
-    lmin = min(lmin, xl[NPL - 1]);
-    lmax = max(lmax, xl[NPL - 1]);
-  }
-  const bool narrow = __all_sync(kFull, hdiff == 0);
-  const uint32_t hmin = ref_y ^ 0x80000000u, hmax = narrow ? hmin : hmin + 1u;
-  const uint32_t k = static_cast<uint32_t>((n - 1) / 2);
-  uint64_t key;
-  if (hmin == hmax) {
-    lmin = __reduce_min_sync(kFull, lmin);
-    lmax = __reduce_max_sync(kFull, lmax);
-    const uint32_t range = lmax - lmin;
-    const int nbits = range ? 32 - __clz(static_cast<int>(range)) : 0;
-    const uint32_t pad = nbits == 32 ? 0xffffffffu : (1u << nbits) - 1u;  // sorts at or after every live value
-#pragma unroll
-    for (int i = 0; i < NPL; ++i) xl[i] = 32 * i < live ? xl[i] - lmin : pad;
-    // candidate slot j: this warp's (already consumed) column slot of tile row j
-    const uint32_t swz = (warp & 1) << 3;
-    auto cand = [&](uint32_t j) {
-      return reinterpret_cast<uint32_t*>(tile + j * 64u + ((((warp >> 1) ^ ((j >> 1) & 3u)) << 4) | swz));
-    };
-    const uint32_t ans = warp_select_bits32<NPL>(xl, nbits, k, hist, lane, cand);
-    key = (static_cast<uint64_t>(hmin) << 32) | (lmin + ans);
-  } else {
-    constexpr uint64_t kSign = 1ull << 63;
-    auto ukey = [&](int i) { return static_cast<uint64_t>(*reinterpret_cast<const int64_t*>(col + i * 2048)) ^ kSign; };
-    uint64_t lo = ~0ull, hi = 0;
-#pragma unroll
-    for (int i = 0; i < NPL; ++i)
-      if (lane + 32 * i < n) {
-        const uint64_t u = ukey(i);
-        lo = u < lo ? u : lo;
-        hi = u > hi ? u : hi;
+  bool issued = blockIdx.x < ntiles;  // (thread 0) the copies of the awaited tile were issued
+  if (threadIdx.x == 0 && issued) issue(blockIdx.x);
+  const unsigned char* col = tile + lane * 64u + ((((warp >> 1) ^ ((lane >> 1) & 3)) << 4) | ((warp & 1) << 3));
+  uint32_t phase = 0;
+  for (int64_t id = blockIdx.x; id < ntiles; id += gridDim.x, phase ^= 1u) {
+    const int64_t w = w0 + id / ngroups;
+    const int64_t c0 = (id % ngroups) * kMedCols;
+    const bool mine = warp < imin64(kMedCols, RS - c0);
+    const int n = static_cast<int>(imin64(W, T - w * W));
+    // a warp goes on only if all its lanes saw the tile (a wait gives up
+    // after its time limit, or at once when another thread has)
+    if (!__all_sync(kFull, mbar_wait_bounded(full, phase, abort))) {
+      if (threadIdx.x == 0) {
+        report(status, SF_ST_TIMEOUT);
+        if (issued) mbar_wait_timeout(full, phase);  // let the copies land before the CTA's memory is released
       }
-    lo = warp_min_u64(lo);
-    hi = warp_max_u64(hi);
-    const uint64_t range = hi - lo;
-    const int nbits = range ? 64 - __clzll(static_cast<long long>(range)) : 0;
-    key = lo + warp_radix_select<uint64_t, NPL>([&](int i) { return ukey(i) - lo; }, n, nbits, k, hist, lane);
+      return;
+    }
+    // Slot i holds a row of the window iff lane + 32 i < n (with kFit, only
+    // the last slot can fail it).  A padding slot repeats a live value; the
+    // high words agree iff their AND equals their OR over the column.
+    auto live = [&](int i) { return (kFit && i + 1 < NPL) || lane + 32 * i < n; };
+    uint32_t xl[NPL];
+    uint32_t hand = 0xffffffffu, hor = 0u, live_x = 0u;
+#pragma unroll
+    for (int i = 0; i < NPL; ++i) {
+      const uint2 v = *reinterpret_cast<const uint2*>(col + i * 2048);  // in the tile even past the window
+      if (i == 0) live_x = kFit && NPL >= 2 ? v.x : __shfl_sync(kFull, v.x, 0);  // row 0 is in every window
+      const bool okr = live(i);
+      xl[i] = okr ? v.x : live_x;
+      hand &= okr ? v.y : 0xffffffffu;
+      hor |= okr ? v.y : 0u;
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(empty);  // this warp is done with the buffer
+    const int64_t next = id + gridDim.x;
+    if (threadIdx.x == 0 && next < ntiles) {
+      issued = mbar_wait_bounded(empty, phase, abort);
+      if (issued) issue(next);  // else the abort flag is set and every warp leaves at its next wait
+    }
+    if (!mine) continue;
+    const uint32_t hw = __reduce_and_sync(kFull, hand);
+    const uint32_t k = static_cast<uint32_t>((n - 1) / 2);
+    if (hw == __reduce_or_sync(kFull, hor)) {
+      uint32_t lmin = xl[0], lmax = xl[0];
+#pragma unroll
+      for (int i = 1; i + 1 < NPL; i += 2) {
+        lmin = __vimin3_u32(lmin, xl[i], xl[i + 1]);
+        lmax = __vimax3_u32(lmax, xl[i], xl[i + 1]);
+      }
+      if ((NPL & 1) == 0) {
+        lmin = min(lmin, xl[NPL - 1]);
+        lmax = max(lmax, xl[NPL - 1]);
+      }
+      lmin = __reduce_min_sync(kFull, lmin);
+      lmax = __reduce_max_sync(kFull, lmax);
+      const uint32_t range = lmax - lmin;
+      const int nbits = range ? 32 - __clz(static_cast<int>(range)) : 0;
+      const uint32_t pad = nbits == 32 ? 0xffffffffu : (1u << nbits) - 1u;  // sorts at or after every live value
+#pragma unroll
+      for (int i = 0; i < NPL; ++i) xl[i] = live(i) ? xl[i] - lmin : pad;
+      const uint32_t ans = warp_select_regs<NPL>(xl, nbits, k, hist, lane);
+      if (lane == 0) m[w * RS + c0 + warp] = static_cast<int64_t>((static_cast<uint64_t>(hw) << 32) | (lmin + ans));
+    } else {
+      // the buffer may already hold the next tile: re-read the column from d
+      const int64_t med = median_column_global<NPL>(d + w * W * RS + c0 + warp, RS, n, hist, lane);
+      if (lane == 0) m[w * RS + c0 + warp] = med;
+    }
   }
-  if (lane == 0) m[w * RS + c0 + warp] = static_cast<int64_t>(key ^ (1ull << 63));
 }
 
 // Windows longer than 1024 steps: the same search, re-reading the column
@@ -673,17 +667,48 @@ cudaError_t launch_median_npl(const int64_t* d, int64_t T, int64_t RS, int64_t W
 }
 
 template <int NPL>
-cudaError_t launch_median_tma(const CUtensorMap& map, int64_t T, int64_t RS, int64_t W, int64_t nW,
-                              int64_t ngroups, int box_rows, int nbox, int64_t* m, uint32_t* status,
+cudaError_t launch_median_tma(const CUtensorMap& map, const int64_t* d, int64_t T, int64_t RS, int64_t W,
+                              int64_t w0, int64_t nW, int64_t n, int64_t ngroups, int box_rows, int nbox, int64_t* m, uint32_t* status,
                               cudaStream_t stream) {
   const size_t tile_rows = std::max<size_t>(size_t(nbox) * box_rows, 32 * NPL);  // every slot's row is in the tile
-  const size_t smem = 1024 + tile_rows * 64 + size_t(kMedCols) * kMedHistWords * 4 + 16;
-  cudaError_t e =
-      cudaFuncSetAttribute(median_tma_kernel<NPL>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  const size_t smem = 1024 + tile_rows * 64 + size_t(kMedCols) * kMedHistWords * 4 + 32;  // + 2 mbarriers, flag
+  auto kern = n > 32 * (NPL - 1) ? median_persist_kernel<NPL, true> : median_persist_kernel<NPL, false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  median_tma_kernel<NPL><<<static_cast<unsigned>(nW * ngroups), kMedThreads, smem, stream>>>(
-      map, T, RS, W, ngroups, box_rows, nbox, static_cast<int>(tile_rows), m, status);
+  int per_sm = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMedThreads, smem);
+  if (e != cudaSuccess) return e;
+  const int64_t grid = std::min<int64_t>(nW * ngroups, int64_t(sm_count()) * std::max(per_sm, 1));
+  count_launch();
+  kern<<<static_cast<unsigned>(grid), kMedThreads, smem, stream>>>(map, d, T, RS, W, w0, nW, ngroups, box_rows,
+                                                                   nbox, m, status);
   return cudaGetLastError();
+}
+
+// Windows [w0, w0 + nW) that each hold n rows: the tensor map's box covers a
+// window in up to four 256-row copies; NPL slots per lane hold n rows.
+cudaError_t launch_median_windows(const int64_t* d, int64_t T, int64_t RS, int64_t W, int64_t w0, int64_t nW,
+                                  int64_t n, int64_t ngroups, int64_t* m, uint32_t* status, cudaStream_t stream,
+                                  bool& done) {
+  done = false;
+  const int nbox = static_cast<int>((n + 255) / 256);
+  const int box_rows = static_cast<int>(((n + nbox - 1) / nbox + 15) / 16 * 16);  // 1024-byte boxes
+  CUtensorMap map;
+  const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(RS), static_cast<cuuint64_t>(T)};
+  const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(RS) * 8};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(kMedCols), static_cast<cuuint32_t>(box_rows)};
+  const cuuint32_t estride[2] = {1, 1};
+  if (encode_fn()(&map, CU_TENSOR_MAP_DATA_TYPE_INT64, 2, const_cast<int64_t*>(d), gdim, gstride, box, estride,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaSuccess;
+  done = true;
+  if (n <= 32) return launch_median_tma<1>(map, d, T, RS, W, w0, nW, n, ngroups, box_rows, nbox, m, status, stream);
+  if (n <= 64) return launch_median_tma<2>(map, d, T, RS, W, w0, nW, n, ngroups, box_rows, nbox, m, status, stream);
+  if (n <= 128) return launch_median_tma<4>(map, d, T, RS, W, w0, nW, n, ngroups, box_rows, nbox, m, status, stream);
+  if (n <= 256) return launch_median_tma<8>(map, d, T, RS, W, w0, nW, n, ngroups, box_rows, nbox, m, status, stream);
+  if (n <= 512) return launch_median_tma<16>(map, d, T, RS, W, w0, nW, n, ngroups, box_rows, nbox, m, status, stream);
+  return launch_median_tma<32>(map, d, T, RS, W, w0, nW, n, ngroups, box_rows, nbox, m, status, stream);
 }
 
 // Self-test of the bounded wait: every thread waits on an mbarrier phase
@@ -726,29 +751,25 @@ cudaError_t launch_window_median(const int64_t* d, int64_t T, int64_t R, int64_t
   const int64_t nW = (T + W - 1) / W;
   const int64_t ngroups = (RS + kMedCols - 1) / kMedCols;
   const int64_t n = std::min(W, T);
-  count_launch();
   // Bulk-copy path: rows of d are 16-byte multiples (RS even), d is 16-byte
   // aligned, windows fit the register path, the driver encoder is available.
+  // A launch's windows share one row count (the slot tests depend on it), so
+  // a short last window gets its own launch.
   if (RS % 2 == 0 && reinterpret_cast<uintptr_t>(d) % 16 == 0 && n <= 1024 && T < (int64_t(1) << 31) &&
       encode_fn() != nullptr) {
-    const int nbox = static_cast<int>((n + 255) / 256);
-    const int box_rows = static_cast<int>(((n + nbox - 1) / nbox + 15) / 16 * 16);  // 1024-byte boxes
-    CUtensorMap map;
-    const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(RS), static_cast<cuuint64_t>(T)};
-    const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(RS) * 8};
-    const cuuint32_t box[2] = {static_cast<cuuint32_t>(kMedCols), static_cast<cuuint32_t>(box_rows)};
-    const cuuint32_t estride[2] = {1, 1};
-    if (encode_fn()(&map, CU_TENSOR_MAP_DATA_TYPE_INT64, 2, const_cast<int64_t*>(d), gdim, gstride, box, estride,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS) {
-      if (n <= 32) return launch_median_tma<1>(map, T, RS, W, nW, ngroups, box_rows, nbox, m, status, stream);
-      if (n <= 64) return launch_median_tma<2>(map, T, RS, W, nW, ngroups, box_rows, nbox, m, status, stream);
-      if (n <= 128) return launch_median_tma<4>(map, T, RS, W, nW, ngroups, box_rows, nbox, m, status, stream);
-      if (n <= 256) return launch_median_tma<8>(map, T, RS, W, nW, ngroups, box_rows, nbox, m, status, stream);
-      if (n <= 512) return launch_median_tma<16>(map, T, RS, W, nW, ngroups, box_rows, nbox, m, status, stream);
-      return launch_median_tma<32>(map, T, RS, W, nW, ngroups, box_rows, nbox, m, status, stream);
+    const int64_t n_last = T - (nW - 1) * W;
+    const int64_t nW_first = n_last == n ? nW : nW - 1;
+    bool done = false;
+    cudaError_t e = launch_median_windows(d, T, RS, W, 0, nW_first, n, ngroups, m, status, stream, done);
+    if (e != cudaSuccess) return e;
+    if (done && nW_first == nW) return cudaSuccess;
+    if (done) {
+      e = launch_median_windows(d, T, RS, W, nW - 1, 1, n_last, ngroups, m, status, stream, done);
+      if (e != cudaSuccess || done) return e;
     }
+    // no tensor map: every window goes the plain-load way below
   }
+  count_launch();
   if (n <= 32) return launch_median_npl<1>(d, T, RS, W, nW, ngroups, m, stream);
   if (n <= 64) return launch_median_npl<2>(d, T, RS, W, nW, ngroups, m, stream);
   if (n <= 128) return launch_median_npl<4>(d, T, RS, W, nW, ngroups, m, stream);

@@ -152,7 +152,8 @@ def test_topk_parity(sf, nW, S, R, k):
 @pytest.mark.parametrize("T,R,S,W", [(7, 3, 5, 1), (9, 4, 3, 2), (33, 2, 3, 3),
                                      (100, 8, 6, 100), (250, 4, 3, 32), (130, 5, 4, 64), (300, 2, 8, 128),
                                      (700, 3, 2, 256), (1100, 2, 4, 512), (2100, 1, 4, 1000),
-                                     (2200, 2, 2, 1024), (2500, 1, 3, 1100), (45, 1024, 10, 20)])
+                                     (2200, 2, 2, 1024), (2500, 1, 3, 1100), (45, 1024, 10, 20),
+                                     (1200, 3, 2, 1000), (600, 2, 3, 200), (1990, 2, 4, 995)])
 @pytest.mark.parametrize("kind", ["ties", "lognormal", "wide", "zeros", "ranges", "clusters"])
 def test_median_parity(sf, T, R, S, W, kind):
     rng = np.random.default_rng(T + W)
