@@ -47,9 +47,11 @@ constexpr int kR0MaxRows = kR0StageBytes / kRowBytes;   // 96 rows
 constexpr int kR1Stages = 6;
 constexpr int kR1StageBytes = kRingBytes / kR1Stages;  // 32 KB
 constexpr int kR1MaxRows = kR1StageBytes / kRowBytes;   // 256 rows (the TMA box limit)
-// The evidence pass streams the window medians m next to d: each 32 KB stage
-// holds a d tile in its first half and the matching m tile in its second.
-constexpr int kR1GainMaxRows = kR1MaxRows / 2;
+// The evidence pass streams the window medians m next to d (regime 1 only):
+// 3 stages of 64 KB, each a 32 KB d tile and the matching 32 KB m tile.
+constexpr int kR1GainStages = 3;
+constexpr int kR1GainStageBytes = kRingBytes / kR1GainStages;  // 64 KB
+constexpr int kR1GainMaxRows = kR1MaxRows;
 constexpr int kMaxStages = kR0Stages;
 constexpr int kRedPerWarp = 64;                       // per-warp partials of one step (<= 2S + 1)
 constexpr int kRedSlots = 2 * kConsumerWarps * kRedPerWarp;  // double-buffered
@@ -78,6 +80,7 @@ struct Params {
   uint64_t* quality;
   uint32_t* status;
   int m_by_tma;  // evidence pass, regime 1: m tiles arrive through the ring
+  int nst, stage_bytes;  // ring stages in use and their size
   // routing-baseline pass
   const int64_t* d;
   int64_t* bM;
@@ -476,20 +479,17 @@ __device__ __forceinline__ void load_global_row(const int64_t* src, int64_t (&v)
 
 
 // Ring stage and phase parity of the j-th tile a CTA streams.
-__device__ __forceinline__ void stage_of(int regime, uint32_t j, uint32_t& st, uint32_t& ph) {
-  if (regime == 0) {  // tile j belongs to warp j % 8, which alternates its two stages
+__device__ __forceinline__ void stage_of(const Params& p, uint32_t j, uint32_t& st, uint32_t& ph) {
+  if (p.regime == 0) {  // tile j belongs to warp j % 8, which alternates its two stages
     const uint32_t i = j / kConsumerWarps;
     st = 2u * (j % kConsumerWarps) + (i & 1u);
     ph = (i >> 1) & 1u;
   } else {
-    st = j % kR1Stages;
-    ph = (j / kR1Stages) & 1u;
+    st = j % static_cast<uint32_t>(p.nst);
+    ph = (j / static_cast<uint32_t>(p.nst)) & 1u;
   }
 }
 
-__device__ __forceinline__ size_t stage_bytes(int regime) {
-  return regime == 0 ? size_t(kR0StageBytes) : size_t(kR1StageBytes);
-}
 
 __device__ void produce(const CUtensorMap* map, const CUtensorMap* map_m, const Params& p, int64_t t_begin,
                         int64_t t_end, unsigned char* ring, uint64_t* full, uint64_t* empty,
@@ -501,15 +501,15 @@ __device__ void produce(const CUtensorMap* map, const CUtensorMap* map_m, const 
   bool ok = true;
   auto issue = [&](int64_t row, int64_t mrow) {
     uint32_t st, ph;
-    stage_of(p.regime, j, st, ph);
+    stage_of(p, j, st, ph);
     if (!mbar_wait_bounded(&empty[st], ph ^ 1u, abort)) {
       ok = false;
       return;
     }
-    unsigned char* dst = ring + size_t(st) * stage_bytes(p.regime);
+    unsigned char* dst = ring + size_t(st) * p.stage_bytes;
     mbar_arrive_expect_tx(&full[st], p.m_by_tma ? 2u * bytes : bytes);
     tma_load_2d(dst, map, 0, static_cast<int32_t>(row), &full[st]);
-    if (p.m_by_tma) tma_load_2d(dst + kR1StageBytes / 2, map_m, 0, static_cast<int32_t>(mrow), &full[st]);
+    if (p.m_by_tma) tma_load_2d(dst + p.stage_bytes / 2, map_m, 0, static_cast<int32_t>(mrow), &full[st]);
     ++j;
   };
   if (p.regime == 0) {
@@ -522,10 +522,10 @@ __device__ void produce(const CUtensorMap* map, const CUtensorMap* map_m, const 
       }
   }
   // copies still in flight: at most one per stage, the last tiles issued
-  const uint32_t nst = p.regime == 0 ? kR0Stages : kR1Stages;
+  const uint32_t nst = static_cast<uint32_t>(p.nst);
   for (uint32_t i = j > nst ? j - nst : 0; i < j; ++i) {
     uint32_t st, ph;
-    stage_of(p.regime, i, st, ph);
+    stage_of(p, i, st, ph);
     mbar_wait_timeout(&full[st], ph);
   }
 }
@@ -678,9 +678,10 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
       else if constexpr (BASE) br.init();
       else fr.init();
       for (int k = 0; k < p.tiles_per_step; ++k, ++j) {
-        const uint32_t st = j % kR1Stages, ph = (j / kR1Stages) & 1u;
+        const uint32_t nst = static_cast<uint32_t>(p.nst);
+        const uint32_t st = j % nst, ph = (j / nst) & 1u;
         const bool have = mbar_wait_bounded(&full[st], ph, abort);
-        const unsigned char* tile = ring + size_t(st) * kR1StageBytes;
+        const unsigned char* tile = ring + size_t(st) * p.stage_bytes;
         const int64_t row0 = min(int64_t(k) * p.box_rows, p.step_rows - p.box_rows);
         const int rank_tile0 = static_cast<int>(row0 * 16 / S);
         const int rank_fresh = static_cast<int>(int64_t(k) * p.box_rows * 16 / S);
@@ -701,13 +702,24 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
                 }
             }
           } else {
-            for (int r = rank_fresh + ctid; r < rank_end; r += kConsumerThreads) {
-              int64_t v[S], mr[S];
-              load_row<S, kSwz>(tile, r - rank_tile0, v);
-              load_row<S, kSwz>(tile + kR1StageBytes / 2, r - rank_tile0, mr);  // m tile of the same ranks
-              const int64_t total = gr.row(v, mr, r, dor, tor);
-              if (p.quality)
-                qual_row(p, qa, t, r, total, p.other_stage >= 0 ? pick<S>(v, p.other_stage) : 0, dor);
+            constexpr int UG = 1;  // rank rows in flight per thread
+            for (int r0 = rank_fresh + ctid; r0 < rank_end; r0 += kConsumerThreads * UG) {
+              int64_t v[UG][S], mr[UG][S];
+#pragma unroll
+              for (int u = 0; u < UG; ++u)
+                if (r0 + kConsumerThreads * u < rank_end) {
+                  const int q = r0 + kConsumerThreads * u - rank_tile0;
+                  load_row<S, kSwz>(tile, q, v[u]);
+                  load_row<S, kSwz>(tile + p.stage_bytes / 2, q, mr[u]);  // m tile of the same ranks
+                }
+#pragma unroll
+              for (int u = 0; u < UG; ++u)
+                if (r0 + kConsumerThreads * u < rank_end) {
+                  const int r = r0 + kConsumerThreads * u;
+                  const int64_t total = gr.row(v[u], mr[u], r, dor, tor);
+                  if (p.quality)
+                    qual_row(p, qa, t, r, total, p.other_stage >= 0 ? pick<S>(v[u], p.other_stage) : 0, dor);
+                }
             }
           }
         }
@@ -1000,6 +1012,8 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
     if (encode(&map, j.d, rows_total) != CUDA_SUCCESS) return cudaErrorInvalidValue;
     map_m = map;
     p.m_by_tma = (j.gain && p.regime == 1) ? 1 : 0;
+    p.nst = p.regime == 0 ? kR0Stages : p.m_by_tma ? kR1GainStages : kR1Stages;
+    p.stage_bytes = p.regime == 0 ? kR0StageBytes : p.m_by_tma ? kR1GainStageBytes : kR1StageBytes;
     if (p.m_by_tma) {
       const int64_t nW = (j.T + j.W - 1) / j.W;
       if (nW * step_rows > int64_t(0x7fffffff) || encode(&map_m, j.m, nW * step_rows) != CUDA_SUCCESS)
