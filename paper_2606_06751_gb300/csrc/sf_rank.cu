@@ -38,6 +38,7 @@ constexpr int kEncThreads = 256;
 constexpr int kEncRows = 1024;  // rank rows per encode item (4 per thread)
 constexpr int kSelThreads = 128;
 constexpr int kSelWarps = kSelThreads / 32;
+constexpr int kSelPerSM = 1536 / kSelThreads;  // resident select CTAs per SM
 constexpr int kSelCand = 2048;  // candidate keys a column may keep after the second pass
 constexpr size_t kRkChunkTarget = size_t(40) << 20;  // scratch of one chunk buffer; two fit L2
 
@@ -351,7 +352,7 @@ struct SelShared {
   int64_t wmin[kSelWarps], wmax[kSelWarps], wsec[kSelWarps];  // 64-bit path
   int64_t lo64;
   uint64_t pref64;
-  uint32_t lo, hi, pref, rem, ncand, bad, sec_key;
+  uint32_t lo, hi, pref, rem, ncand, bad, sec_key, kept;
   int nb, compact, bytes64;
   int64_t med, F, sec;
 };
@@ -434,7 +435,54 @@ __device__ __noinline__ void select_column_64(const RankParams& p, int64_t t, in
   __syncthreads();
 }
 
-__global__ void __launch_bounds__(kSelThreads, 12) rank_select_kernel(const RankParams p) {
+// The first pass of a column's selection resolves kWideBits bits at once, in
+// a 2^kWideBits-bin histogram that lives in the candidate slots (unused
+// until the next pass).
+constexpr int kWideBits = 11;
+constexpr int kWideBins = 1 << kWideBits;
+static_assert(kWideBins <= kSelCand, "the wide histogram lives in the candidate slots");
+
+// The bin of a 2048-bin shared-memory histogram (16-byte aligned) that holds
+// rank `rem`, and the count below it: each lane sums 64 consecutive bins, one
+// warp scan picks the owning lane, and the owner's 64 bins are split two per
+// lane for a second scan.  Whole warp; results in every lane.
+__device__ __forceinline__ void hist_find_wide(const uint32_t* h, uint32_t rem, int lane, uint32_t& digit,
+                                               uint32_t& below) {
+  const uint4* h4 = reinterpret_cast<const uint4*>(h) + 16 * lane;
+  uint32_t sum = 0;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const uint4 v = h4[j];
+    sum += v.x + v.y + v.z + v.w;
+  }
+  uint32_t incl = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t up = __shfl_up_sync(kFull, incl, o);
+    if (lane >= o) incl += up;
+  }
+  const uint32_t excl = incl - sum;
+  const int owner = __ffs(__ballot_sync(kFull, excl <= rem && rem < incl)) - 1;
+  const uint32_t base = __shfl_sync(kFull, excl, owner);
+  const uint32_t r = rem - base;  // rank within the owner's 64 bins
+  const uint2 pr = reinterpret_cast<const uint2*>(h + 64 * owner)[lane];
+  const uint32_t two = pr.x + pr.y;
+  uint32_t in2 = two;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t up = __shfl_up_sync(kFull, in2, o);
+    if (lane >= o) in2 += up;
+  }
+  const uint32_t ex2 = in2 - two;
+  const int sub = __ffs(__ballot_sync(kFull, ex2 <= r && r < in2)) - 1;
+  const uint32_t e2 = __shfl_sync(kFull, ex2, sub);
+  const uint32_t x = __shfl_sync(kFull, pr.x, sub);
+  const bool second = r - e2 >= x;  // past the pair's first bin
+  digit = 64u * owner + 2u * sub + (second ? 1u : 0u);
+  below = base + e2 + (second ? x : 0u);
+}
+
+__global__ void __launch_bounds__(kSelThreads, kSelPerSM) rank_select_kernel(const RankParams p) {
   __shared__ __align__(16) SelShared sh;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int S = static_cast<int>(p.S);
@@ -485,34 +533,76 @@ __global__ void __launch_bounds__(kSelThreads, 12) rank_select_kernel(const Rank
     } else {
       const uint32_t lo = sh.lo;
       const int nb = sh.nb;
-      // ---- first pass: every key counts (the top digit), four keys per load
+      // ---- first pass: every key counts; the top kWideBits bits of the range
+      // go into the wide histogram (the candidate slots), four keys per load
+      int start_hi = 0;  // bits still to resolve after the first pass
       if (nb > 0) {
-        for (int i = tid; i < 256; i += kSelThreads) sh.hist[i] = 0;
+        const int shift = nb > kWideBits ? nb - kWideBits : 0;  // offsets are below 2^nb
+        uint32_t* wide = sh.cand;
+        for (int i = tid; i < kWideBins / 4; i += kSelThreads)
+          reinterpret_cast<uint4*>(wide)[i] = make_uint4(0, 0, 0, 0);
         __syncthreads();
-        const int shift = nb > 8 ? nb - 8 : 0;  // offsets are below 2^nb; the mask only guards the bins
         const int nq = R >> 2;
         for (int i = tid; i < nq; i += kSelThreads) {
           const uint4 k4 = reinterpret_cast<const uint4*>(col)[i];
-          atomicAdd(&sh.hist[((k4.x - lo) >> shift) & 255u], 1u);
-          atomicAdd(&sh.hist[((k4.y - lo) >> shift) & 255u], 1u);
-          atomicAdd(&sh.hist[((k4.z - lo) >> shift) & 255u], 1u);
-          atomicAdd(&sh.hist[((k4.w - lo) >> shift) & 255u], 1u);
+          atomicAdd(&wide[((k4.x - lo) >> shift) & (kWideBins - 1)], 1u);
+          atomicAdd(&wide[((k4.y - lo) >> shift) & (kWideBins - 1)], 1u);
+          atomicAdd(&wide[((k4.z - lo) >> shift) & (kWideBins - 1)], 1u);
+          atomicAdd(&wide[((k4.w - lo) >> shift) & (kWideBins - 1)], 1u);
         }
-        for (int r = 4 * nq + tid; r < R; r += kSelThreads) atomicAdd(&sh.hist[((col[r] - lo) >> shift) & 255u], 1u);
+        for (int r = 4 * nq + tid; r < R; r += kSelThreads)
+          atomicAdd(&wide[((col[r] - lo) >> shift) & (kWideBins - 1)], 1u);
         __syncthreads();
         if (warp == 0) {
           uint32_t digit, below;
-          hist_find(sh.hist, sh.rem, lane, digit, below);
+          hist_find_wide(wide, sh.rem, lane, digit, below);
           if (lane == 0) {
             sh.pref = digit << shift;
             sh.rem -= below;
-            sh.compact = nb > 8 && sh.hist[digit] <= kSelCand;
+            sh.kept = wide[digit];
+            sh.compact = shift > 0 && wide[digit] <= kSelCand;
           }
+        }
+        __syncthreads();
+        start_hi = shift;
+        if (shift > 0 && sh.kept <= 32) {
+          // ---- at most 32 keys share the chosen bin: gather them (the
+          // wide histogram is dead) and rank them by counting in one warp
+          __syncthreads();  // every thread has read kept
+          if (tid == 0) sh.ncand = 0;
+          __syncthreads();
+          const uint32_t dsel = sh.pref >> shift;
+          auto gather = [&](uint32_t k) {
+            if (((k - lo) >> shift) == dsel) sh.cand[atomicAdd(&sh.ncand, 1u)] = k - lo;
+          };
+          for (int i = tid; i < nq; i += kSelThreads) {
+            const uint4 k4 = reinterpret_cast<const uint4*>(col)[i];
+            gather(k4.x);
+            gather(k4.y);
+            gather(k4.z);
+            gather(k4.w);
+          }
+          for (int r = 4 * nq + tid; r < R; r += kSelThreads) gather(col[r]);
+          __syncthreads();
+          if (warp == 0) {
+            const uint32_t kept = sh.kept, rem = sh.rem;
+            const uint32_t v = static_cast<uint32_t>(lane) < kept ? sh.cand[lane] : 0xffffffffu;
+            uint32_t lt = 0, le = 0;
+            for (uint32_t q = 0; q < kept; ++q) {
+              const uint32_t c = __shfl_sync(kFull, v, static_cast<int>(q));
+              lt += c < v ? 1u : 0u;
+              le += c <= v ? 1u : 0u;
+            }
+            const uint32_t hit = __ballot_sync(kFull, static_cast<uint32_t>(lane) < kept && lt <= rem && rem < le);
+            const uint32_t ans = __shfl_sync(kFull, v, __ffs(hit) - 1);
+            if (lane == 0) sh.pref = ans;
+          }
+          start_hi = 0;
         }
       }
       // ---- later passes: 8 bits each below the top digit
       bool read_all = true;  // the column is still read from L2
-      for (int hi = nb - 8; hi > 0; hi -= 8) {
+      for (int hi = start_hi; hi > 0; hi -= 8) {
         const int shift = hi > 8 ? hi - 8 : 0;
         const uint32_t mask = (1u << (hi - shift)) - 1u;
         __syncthreads();  // the last digit search is done: its pref and rem are visible, hist is free
@@ -752,7 +842,7 @@ cudaError_t launch_rank_select(const int64_t* d, int64_t T, int64_t R, int64_t S
       default: e = launch_encode<0>(p, stream, c == 0); break;
     }
     if (e != cudaSuccess) return e;
-    const int sel_grid = static_cast<int>(std::min<int64_t>(p.Tc * S, int64_t(sms) * 12));
+    const int sel_grid = static_cast<int>(std::min<int64_t>(p.Tc * S, int64_t(sms) * kSelPerSM));
     count_launch();
     if ((e = launch_pdl(rank_select_kernel, sel_grid, kSelThreads, p, stream)) != cudaSuccess) return e;
   }

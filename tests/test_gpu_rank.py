@@ -41,6 +41,10 @@ def make(T, R, S, seed, kind):
         return rng.integers(0, 1 << 41, size=(T, R, S), dtype=np.int64)
     med = rng.uniform(1e6, 5e7, size=S)
     d = np.rint(med * np.exp(0.1 * rng.standard_normal((T, R, S)))).astype(np.int64)
+    if kind == "sampleskew":  # the first 4 ranks of every 32 far faster: a sample of them misleads
+        d[:, (np.arange(R) % 32) < 4, :] //= 4
+    if kind == "cluster":   # 70 % of the values equal: the median sits in one heavy tie
+        d[rng.random((T, R, S)) < 0.7] = int(med[0])
     if kind == "mixed":     # a few steps with a multi-second stall on one rank (64-bit path)
         for t in rng.choice(T, size=max(1, T // 7), replace=False):
             d[t, rng.integers(R), rng.integers(S)] += int(rng.integers(1 << 31, 1 << 33))
@@ -57,7 +61,7 @@ SHAPES = [(20, 1, 1), (9, 2, 3), (37, 3, 5), (11, 7, 32), (6, 5, 18), (50, 2, 8)
 
 
 @pytest.mark.parametrize("T,R,S", SHAPES)
-@pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal", "wide", "mixed"])
+@pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal", "wide", "mixed", "sampleskew", "cluster"])
 def test_rank_lag_parity(sf, T, R, S, kind):
     d_np = make(T, R, S, T * 17 + R * 5 + S, kind)
     o = O.rank_lag(d_np)
@@ -116,6 +120,18 @@ def test_raw_spread_parity(sf, T, R, S, t0, W):
     o = O.raw_spread(d_np, W, t0)
     st = sf.new_status("cuda")
     got = sf.sf_raw_spread(dev(d_np), W, t0=t0, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert np.array_equal(host(got), o)
+
+
+@pytest.mark.parametrize("T,R,S", [(9, 8192, 8), (5, 4096, 3), (3, 65536, 2)])
+@pytest.mark.parametrize("kind", ["sampleskew", "cluster"])
+def test_raw_spread_misleading_sample(sf, T, R, S, kind):
+    d_np = make(T, R, S, T * 3 + R + S, kind)
+    o = O.raw_spread(d_np, 4, 0)
+    st = sf.new_status("cuda")
+    got = sf.sf_raw_spread(dev(d_np), 4, status=st)
     torch.cuda.synchronize()
     assert int(st.item()) == 0
     assert np.array_equal(host(got), o)
