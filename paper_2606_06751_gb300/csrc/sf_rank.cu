@@ -231,6 +231,8 @@ __global__ void __launch_bounds__(kEncThreads) rank_encode_split_kernel(const Ra
   constexpr int kRowsPerPass = kEncThreads / L;  // rows the CTA covers per pass
   constexpr int kUnroll = 4;                     // passes whose loads are in flight together
   constexpr int kWarps = kEncThreads / 32;
+  // values below 2^kNarrowBits: a row's prefixes stay below SC * 2^kNarrowBits <= 2^31
+  constexpr int kNarrowBits = SC <= 4 ? 29 : SC <= 8 ? 28 : 27;
   __shared__ int64_t sref[kRkMaxS];
   __shared__ uint32_t wmn[kWarps][kRkMaxS], wmx[kWarps][kRkMaxS], wm2[kWarps][kRkMaxS];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -259,6 +261,9 @@ __global__ void __launch_bounds__(kEncThreads) rank_encode_split_kernel(const Ra
     }
     __syncthreads();
     const int64_t ref0 = sref[2 * j], ref1 = sref[2 * j + 1];
+    bool ref_narrow = true;  // rank 0's values (or prefixes) all in [0, 2^31)
+#pragma unroll
+    for (int q = 0; q < SC; ++q) ref_narrow &= (static_cast<uint64_t>(sref[q]) >> 31) == 0;
     uint32_t mn0 = 0xffffffffu, a0 = 0u, b0 = 0u, mn1 = 0xffffffffu, a1 = 0u, b1 = 0u;
     bool bad = false;
     const int64_t rb = int64_t(blk) * kEncRows;
@@ -277,8 +282,40 @@ __global__ void __launch_bounds__(kEncThreads) rank_encode_split_kernel(const Ra
       for (int u = 0; u < kUnroll; ++u) {
         const int r = r0 + u * kRowsPerPass + rsub;
         const bool live = r < nrows;
-        dor |= static_cast<uint32_t>(static_cast<uint64_t>(v[u].x) >> 32) |
-               static_cast<uint32_t>(static_cast<uint64_t>(v[u].y) >> 32);
+        const uint32_t hw = static_cast<uint32_t>(static_cast<uint64_t>(v[u].x) >> 32) |
+                            static_cast<uint32_t>(static_cast<uint64_t>(v[u].y) >> 32);
+        // 32-bit arithmetic when every value of the warp's rows is below
+        // 2^kNarrowBits and so is rank 0's row: prefixes then stay below 2^31
+        // and every key difference is exact in 32 bits
+        const bool narrow = __all_sync(kFull, ((hw | ((static_cast<uint32_t>(v[u].x) |
+                                                     static_cast<uint32_t>(v[u].y)) >> kNarrowBits)) == 0) &&
+                                                  ref_narrow);
+        if (narrow) {
+          uint32_t y0 = static_cast<uint32_t>(v[u].x), y1 = static_cast<uint32_t>(v[u].y);
+          if (p.of_prefix) {
+            const uint32_t pair = y0 + y1;
+            uint32_t incl = pair;
+#pragma unroll
+            for (int o = 1; o < L; o <<= 1) {
+              const uint32_t up = __shfl_up_sync(kFull, incl, o, L);
+              if (j >= o) incl += up;
+            }
+            y0 += incl - pair;
+            y1 = incl;
+          }
+          const uint32_t q0 = (y0 - static_cast<uint32_t>(ref0)) ^ 0x80000000u;
+          const uint32_t q1 = (y1 - static_cast<uint32_t>(ref1)) ^ 0x80000000u;
+          if (live) {
+            k0[r] = q0;
+            k1[r] = q1;
+            mn0 = q0 < mn0 ? q0 : mn0;
+            mn1 = q1 < mn1 ? q1 : mn1;
+            top2_merge<uint32_t>(a0, b0, q0, 0u);
+            top2_merge<uint32_t>(a1, b1, q1, 0u);
+          }
+          continue;
+        }
+        dor |= hw;
         int64_t x0 = v[u].x, x1 = v[u].y;
         if (p.of_prefix) {
           // prefix before this pair: scan of the pair sums over the row's lanes

@@ -45,6 +45,11 @@ def make(T, R, S, seed, kind):
         d[:, (np.arange(R) % 32) < 4, :] //= 4
     if kind == "cluster":   # 70 % of the values equal: the median sits in one heavy tie
         d[rng.random((T, R, S)) < 0.7] = int(med[0])
+    if kind == "boundary":  # values around 2^27..2^29: the 32-bit encode's limits for 16, 8 and 4 stages
+        edges = np.array([(1 << b) + o for b in (27, 28, 29) for o in (-2, -1, 0, 1)], dtype=np.int64)
+        return edges[rng.integers(0, len(edges), size=(T, R, S))]
+    if kind == "refwide":   # rank 0 alone far from the rest at one stage
+        d[:, 0, S // 2] += 1 << 31
     if kind == "mixed":     # a few steps with a multi-second stall on one rank (64-bit path)
         for t in rng.choice(T, size=max(1, T // 7), replace=False):
             d[t, rng.integers(R), rng.integers(S)] += int(rng.integers(1 << 31, 1 << 33))
@@ -61,7 +66,8 @@ SHAPES = [(20, 1, 1), (9, 2, 3), (37, 3, 5), (11, 7, 32), (6, 5, 18), (50, 2, 8)
 
 
 @pytest.mark.parametrize("T,R,S", SHAPES)
-@pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal", "wide", "mixed", "sampleskew", "cluster"])
+@pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal", "wide", "mixed", "sampleskew", "cluster", "boundary",
+                                  "refwide"])
 def test_rank_lag_parity(sf, T, R, S, kind):
     d_np = make(T, R, S, T * 17 + R * 5 + S, kind)
     o = O.rank_lag(d_np)
