@@ -15,14 +15,15 @@
 //    walks blocks of 1024 rank rows of one step and writes each block's
 //    minimum, maximum and second largest key per stage and a flag for a value
 //    2^31 or more away from rank 0's (that step then takes the 64-bit path).
+//    A warp whose values are all small works in 32-bit arithmetic.
 //  rank_select_kernel - one CTA per (step, stage) column at a time: radix
-//    selection on the key offsets from the column minimum, the first digit
-//    starting at the highest bit of the range so that it spreads over the 256
-//    bins.  The first pass reads the column from L2 four keys at a time; the
-//    second reads it again, counts the keys in the chosen bin and keeps them
-//    as candidates, so later passes read only those.  Once a column has been
-//    read for the last time its L2 lines are discarded, so the dead scratch
-//    is never written back to HBM.
+//    selection on the key offsets from the column minimum.  The first pass
+//    reads the column from L2 four keys at a time into a 2048-bin histogram
+//    of the top 11 bits of the range.  A chosen bin of at most 32 keys is
+//    gathered by a second read and ranked by counting in one warp; a fuller
+//    bin is kept as candidates by the second read, so later 8-bit passes read
+//    only those.  Once a column has been read for the last time its L2 lines
+//    are discarded, so the dead scratch is never written back to HBM.
 // A last small kernel forms delta-lag from the lag.
 #include <algorithm>
 #include <cstdint>
