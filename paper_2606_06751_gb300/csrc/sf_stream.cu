@@ -23,6 +23,7 @@
 // global loads.  Both paths share the per-step epilogues.
 #include <algorithm>
 #include <numeric>
+#include <type_traits>
 
 #include "sf_device.cuh"
 #include "sf_launch.h"
@@ -81,6 +82,7 @@ struct Params {
   uint32_t* status;
   int m_by_tma;  // evidence pass, regime 1: m tiles arrive through the ring
   int nst, stage_bytes;  // ring stages in use and their size
+  int groups;            // regime 1: consumer warp groups, each taking every groups-th step
   // routing-baseline pass
   const int64_t* d;
   int64_t* bM;
@@ -479,16 +481,26 @@ __device__ __forceinline__ void load_global_row(const int64_t* src, int64_t (&v)
 
 
 // Ring stage and phase parity of the j-th tile a CTA streams.
-__device__ __forceinline__ void stage_of(const Params& p, uint32_t j, uint32_t& st, uint32_t& ph) {
-  if (p.regime == 0) {  // tile j belongs to warp j % 8, which alternates its two stages
-    const uint32_t i = j / kConsumerWarps;
-    st = 2u * (j % kConsumerWarps) + (i & 1u);
-    ph = (i >> 1) & 1u;
-  } else {
-    st = j % static_cast<uint32_t>(p.nst);
-    ph = (j / static_cast<uint32_t>(p.nst)) & 1u;
-  }
+// Regime 0: tile j belongs to warp j % 8, which alternates its two stages.
+__device__ __forceinline__ void stage_of_r0(uint32_t j, uint32_t& st, uint32_t& ph) {
+  const uint32_t i = j / kConsumerWarps;
+  st = 2u * (j % kConsumerWarps) + (i & 1u);
+  ph = (i >> 1) & 1u;
 }
+
+// Regime 1: the steps go to the warp groups in turn; group g owns stages g,
+// g + G, ..., g + G (nst / G - 1) and fills them in that order.  The walk of
+// one group's stages, kept incrementally (no division per tile).
+struct GroupRing {
+  uint32_t slot = 0, ph = 0;  // next stage slot within the group and its phase parity
+  __device__ __forceinline__ uint32_t stage(uint32_t g, uint32_t G) const { return g + G * slot; }
+  __device__ __forceinline__ void advance(uint32_t spg) {
+    if (++slot == spg) {
+      slot = 0;
+      ph ^= 1u;
+    }
+  }
+};
 
 
 __device__ void produce(const CUtensorMap* map, const CUtensorMap* map_m, const Params& p, int64_t t_begin,
@@ -498,14 +510,15 @@ __device__ void produce(const CUtensorMap* map, const CUtensorMap* map_m, const 
   if (p.m_by_tma) prefetch_tensormap(map_m);
   const uint32_t bytes = static_cast<uint32_t>(p.box_rows) * kRowBytes;
   uint32_t j = 0;  // tiles issued
+  uint32_t used = 0, last_ph = 0;  // per stage: issued into at all, parity of the last issue
   bool ok = true;
-  auto issue = [&](int64_t row, int64_t mrow) {
-    uint32_t st, ph;
-    stage_of(p, j, st, ph);
+  auto issue = [&](int64_t row, int64_t mrow, uint32_t st, uint32_t ph) {
     if (!mbar_wait_bounded(&empty[st], ph ^ 1u, abort)) {
       ok = false;
       return;
     }
+    used |= 1u << st;
+    last_ph = (last_ph & ~(1u << st)) | (ph << st);
     unsigned char* dst = ring + size_t(st) * p.stage_bytes;
     mbar_arrive_expect_tx(&full[st], p.m_by_tma ? 2u * bytes : bytes);
     tma_load_2d(dst, map, 0, static_cast<int32_t>(row), &full[st]);
@@ -513,21 +526,42 @@ __device__ void produce(const CUtensorMap* map, const CUtensorMap* map_m, const 
     ++j;
   };
   if (p.regime == 0) {
-    for (int64_t t = t_begin; t < t_end && ok; t += p.K) issue(t * p.step_rows, 0);
-  } else {
+    for (int64_t t = t_begin; t < t_end && ok; t += p.K) {
+      uint32_t st, ph;
+      stage_of_r0(j, st, ph);
+      issue(t * p.step_rows, 0, st, ph);
+    }
+  } else if (p.groups == 1) {
+    GroupRing rg;
+    const uint32_t nst = static_cast<uint32_t>(p.nst);
     for (int64_t t = t_begin; t < t_end && ok; ++t)
       for (int k = 0; k < p.tiles_per_step && ok; ++k) {
         const int64_t r0 = min(int64_t(k) * p.box_rows, p.step_rows - p.box_rows);
-        issue(t * p.step_rows + r0, (t / p.W) * p.step_rows + r0);
+        issue(t * p.step_rows + r0, (t / p.W) * p.step_rows + r0, rg.slot, rg.ph);
+        rg.advance(nst);
       }
+  } else {
+    const uint32_t G = static_cast<uint32_t>(p.groups), spg = static_cast<uint32_t>(p.nst) / G;
+    uint32_t walk = 0;  // per group g (<= 4): bits 4g..4g+2 the next stage slot, bit 4g+3 its phase
+    uint32_t g = 0;     // the group of step t
+    for (int64_t t = t_begin; t < t_end && ok; ++t) {
+      const uint32_t sh = 4u * g;
+      uint32_t slot = (walk >> sh) & 7u, ph = (walk >> (sh + 3)) & 1u;
+      for (int k = 0; k < p.tiles_per_step && ok; ++k) {
+        const int64_t r0 = min(int64_t(k) * p.box_rows, p.step_rows - p.box_rows);
+        issue(t * p.step_rows + r0, (t / p.W) * p.step_rows + r0, g + G * slot, ph);
+        if (++slot == spg) {
+          slot = 0;
+          ph ^= 1u;
+        }
+      }
+      walk = (walk & ~(15u << sh)) | (slot << sh) | (ph << (sh + 3));
+      g = g + 1 == G ? 0 : g + 1;
+    }
   }
-  // copies still in flight: at most one per stage, the last tiles issued
-  const uint32_t nst = static_cast<uint32_t>(p.nst);
-  for (uint32_t i = j > nst ? j - nst : 0; i < j; ++i) {
-    uint32_t st, ph;
-    stage_of(p, i, st, ph);
-    mbar_wait_timeout(&full[st], ph);
-  }
+  // copies still in flight: at most one per stage, the last issued into it
+  for (uint32_t st = 0; st < kMaxStages; ++st)
+    if ((used >> st) & 1u) mbar_wait_timeout(&full[st], (last_ph >> st) & 1u);
 }
 
 // --------------------------------------------------------------------------
@@ -554,7 +588,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
   if (threadIdx.x == 0) {
     for (int i = 0; i < kMaxStages; ++i) {
       mbar_init(&full[i], 1);
-      mbar_init(&empty[i], p.regime == 0 ? 1u : uint32_t(kConsumerWarps));
+      mbar_init(&empty[i], p.regime == 0 ? 1u : uint32_t(kConsumerWarps / p.groups));
     }
     *abort = 0;
     fence_barrier_init();
@@ -664,122 +698,139 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
       if (lane == 0) mbar_arrive(&empty[st]);
     }
   } else {
-    // ---- one step per CTA, tiles_per_step tiles per step
-    const int ctid = threadIdx.x;
-    uint32_t j = 0;
-    int buf = 0;
-    for (int64_t t = t_begin; t < t_end; ++t) {
-      const int64_t w = GAIN ? t / p.W : 0;
-      if (GAIN && p.quality) qual_window(p, qa, w, lane);
-      FrontierRows<S> fr;
-      GainRows<S> gr;
-      BaseRows<S> br;
-      if constexpr (GAIN) gr.init();
-      else if constexpr (BASE) br.init();
-      else fr.init();
-      for (int k = 0; k < p.tiles_per_step; ++k, ++j) {
-        const uint32_t nst = static_cast<uint32_t>(p.nst);
-        const uint32_t st = j % nst, ph = (j / nst) & 1u;
-        const bool have = mbar_wait_bounded(&full[st], ph, abort);
-        const unsigned char* tile = ring + size_t(st) * p.stage_bytes;
-        const int64_t row0 = min(int64_t(k) * p.box_rows, p.step_rows - p.box_rows);
-        const int rank_tile0 = static_cast<int>(row0 * 16 / S);
-        const int rank_fresh = static_cast<int>(int64_t(k) * p.box_rows * 16 / S);
-        const int rank_end = static_cast<int>((row0 + p.box_rows) * 16 / S);
-        if (have) {
-          if constexpr (!GAIN) {
-            for (int r0 = rank_fresh + ctid; r0 < rank_end; r0 += kConsumerThreads * U) {
-              int64_t v[U][S];
-#pragma unroll
-              for (int u = 0; u < U; ++u)
-                if (r0 + kConsumerThreads * u < rank_end)
-                  load_row<S, kSwz>(tile, r0 + kConsumerThreads * u - rank_tile0, v[u]);
-#pragma unroll
-              for (int u = 0; u < U; ++u)
-                if (r0 + kConsumerThreads * u < rank_end) {
-                  if constexpr (BASE) br.row(v[u], r0 + kConsumerThreads * u, dor, tor);
-                  else fr.row(v[u], r0 + kConsumerThreads * u, dor, tor);
-                }
+    // ---- one step per warp group (of kConsumerWarps / groups warps), the
+    // groups taking steps in turn, tiles_per_step tiles per step
+    // (the group count is a compile-time constant in each copy of the loop)
+    auto consume = [&](auto ng) {
+      constexpr int NG = decltype(ng)::value;
+      constexpr int gw = kConsumerWarps / NG;  // warps per group
+      const int g = warp / gw, lw = warp % gw;
+      constexpr int gthreads = gw * 32;
+      const int ctid = threadIdx.x - g * gthreads;  // thread within the group
+      const uint32_t spg = static_cast<uint32_t>(p.nst / NG);  // stages of this group
+      GroupRing gring;
+      int buf = 0;
+      for (int64_t t = t_begin + g; t < t_end; t += NG) {
+        const int64_t w = GAIN ? t / p.W : 0;
+        if (GAIN && p.quality) qual_window(p, qa, w, lane);
+        [[maybe_unused]] FrontierRows<S> fr;
+        [[maybe_unused]] GainRows<S> gr;
+        [[maybe_unused]] BaseRows<S> br;
+        if constexpr (GAIN) gr.init();
+        else if constexpr (BASE) br.init();
+        else fr.init();
+        for (int k = 0; k < p.tiles_per_step; ++k) {
+          const uint32_t st = gring.stage(g, NG), ph = gring.ph;
+          gring.advance(spg);
+          const bool have = mbar_wait_bounded(&full[st], ph, abort);
+          const unsigned char* tile = ring + size_t(st) * p.stage_bytes;
+          const int64_t row0 = min(int64_t(k) * p.box_rows, p.step_rows - p.box_rows);
+          const int rank_tile0 = static_cast<int>(row0 * 16 / S);
+          const int rank_fresh = static_cast<int>(int64_t(k) * p.box_rows * 16 / S);
+          const int rank_end = static_cast<int>((row0 + p.box_rows) * 16 / S);
+          if (have) {
+            if constexpr (!GAIN) {
+              for (int r0 = rank_fresh + ctid; r0 < rank_end; r0 += gthreads * U) {
+                int64_t v[U][S];
+  #pragma unroll
+                for (int u = 0; u < U; ++u)
+                  if (r0 + gthreads * u < rank_end) load_row<S, kSwz>(tile, r0 + gthreads * u - rank_tile0, v[u]);
+  #pragma unroll
+                for (int u = 0; u < U; ++u)
+                  if (r0 + gthreads * u < rank_end) {
+                    if constexpr (BASE) br.row(v[u], r0 + gthreads * u, dor, tor);
+                    else fr.row(v[u], r0 + gthreads * u, dor, tor);
+                  }
+              }
+            } else {
+              constexpr int UG = 1;  // rank rows in flight per thread
+              for (int r0 = rank_fresh + ctid; r0 < rank_end; r0 += gthreads * UG) {
+                int64_t v[UG][S], mr[UG][S];
+  #pragma unroll
+                for (int u = 0; u < UG; ++u)
+                  if (r0 + gthreads * u < rank_end) {
+                    const int q = r0 + gthreads * u - rank_tile0;
+                    load_row<S, kSwz>(tile, q, v[u]);
+                    load_row<S, kSwz>(tile + p.stage_bytes / 2, q, mr[u]);  // m tile of the same ranks
+                  }
+  #pragma unroll
+                for (int u = 0; u < UG; ++u)
+                  if (r0 + gthreads * u < rank_end) {
+                    const int r = r0 + gthreads * u;
+                    const int64_t total = gr.row(v[u], mr[u], r, dor, tor);
+                    if (p.quality)
+                      qual_row(p, qa, t, r, total, p.other_stage >= 0 ? pick<S>(v[u], p.other_stage) : 0, dor);
+                  }
+              }
+            }
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&empty[st]);
+        }
+        // cross-rank reduction: warp redux, then one exchange through shared memory
+        uint64_t* slot = red + (buf * kConsumerWarps + warp) * kRedPerWarp;
+        uint64_t bslow = 0;
+        if constexpr (BASE) bslow = warp_max_u64(br.slow);
+  #pragma unroll
+        for (int s = 0; s < S; ++s) {
+          if constexpr (MODE == 0) {
+            const uint64_t km = warp_max_u64(fr.key(s));
+            if (lane == s) slot[s] = km;
+          } else if constexpr (BASE) {
+            const uint64_t mx = warp_max_u64(static_cast<uint64_t>(br.mx[s]));
+            const uint64_t sm = warp_sum_u64(br.sm[s]);
+            if (lane == s) {
+              slot[s] = mx;
+              slot[S + s] = sm;
             }
           } else {
-            constexpr int UG = 1;  // rank rows in flight per thread
-            for (int r0 = rank_fresh + ctid; r0 < rank_end; r0 += kConsumerThreads * UG) {
-              int64_t v[UG][S], mr[UG][S];
-#pragma unroll
-              for (int u = 0; u < UG; ++u)
-                if (r0 + kConsumerThreads * u < rank_end) {
-                  const int q = r0 + kConsumerThreads * u - rank_tile0;
-                  load_row<S, kSwz>(tile, q, v[u]);
-                  load_row<S, kSwz>(tile + p.stage_bytes / 2, q, mr[u]);  // m tile of the same ranks
-                }
-#pragma unroll
-              for (int u = 0; u < UG; ++u)
-                if (r0 + kConsumerThreads * u < rank_end) {
-                  const int r = r0 + kConsumerThreads * u;
-                  const int64_t total = gr.row(v[u], mr[u], r, dor, tor);
-                  if (p.quality)
-                    qual_row(p, qa, t, r, total, p.other_stage >= 0 ? pick<S>(v[u], p.other_stage) : 0, dor);
-                }
+            const uint64_t f = warp_max_u64(gr.key(s));
+            const uint64_t g = warp_max_u64(gr.G(s));
+            if (lane == s) {
+              slot[s] = f;
+              slot[S + s] = g;
             }
           }
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&empty[st]);
-      }
-      // cross-rank reduction: warp redux, then one exchange through shared memory
-      uint64_t* slot = red + (buf * kConsumerWarps + warp) * kRedPerWarp;
-      uint64_t bslow = 0;
-      if constexpr (BASE) bslow = warp_max_u64(br.slow);
-#pragma unroll
-      for (int s = 0; s < S; ++s) {
-        if constexpr (MODE == 0) {
-          const uint64_t km = warp_max_u64(fr.key(s));
-          if (lane == s) slot[s] = km;
-        } else if constexpr (BASE) {
-          const uint64_t mx = warp_max_u64(static_cast<uint64_t>(br.mx[s]));
-          const uint64_t sm = warp_sum_u64(br.sm[s]);
-          if (lane == s) {
-            slot[s] = mx;
-            slot[S + s] = sm;
-          }
-        } else {
-          const uint64_t f = warp_max_u64(gr.key(s));
-          const uint64_t g = warp_max_u64(gr.G(s));
-          if (lane == s) {
-            slot[s] = f;
-            slot[S + s] = g;
-          }
+        if (BASE && lane == 0) slot[2 * S] = bslow;
+        // the group's own barrier, its id an immediate operand
+        switch (g) {
+          case 0: named_barrier(1, gthreads); break;
+          case 1: named_barrier(2, gthreads); break;
+          case 2: named_barrier(3, gthreads); break;
+          default: named_barrier(4, gthreads); break;
         }
-      }
-      if (BASE && lane == 0) slot[2 * S] = bslow;
-      named_barrier(1, kConsumerThreads);
-      if (warp == 0) {
-        uint64_t v0 = 0, v1 = 0, v2 = 0;
-        if (lane < S) {
-#pragma unroll
-          for (int ww = 0; ww < kConsumerWarps; ++ww) {
-            const uint64_t* sl = red + (buf * kConsumerWarps + ww) * kRedPerWarp;
-            v0 = sl[lane] > v0 ? sl[lane] : v0;
-            if (GAIN) v1 = sl[S + lane] > v1 ? sl[S + lane] : v1;
-            if (BASE) v1 += sl[S + lane];
+        if (lw == 0) {
+          uint64_t v0 = 0, v1 = 0, v2 = 0;
+          if (lane < S) {
+            for (int ww = warp; ww < warp + gw; ++ww) {
+              const uint64_t* sl = red + (buf * kConsumerWarps + ww) * kRedPerWarp;
+              v0 = sl[lane] > v0 ? sl[lane] : v0;
+              if (GAIN) v1 = sl[S + lane] > v1 ? sl[S + lane] : v1;
+              if (BASE) v1 += sl[S + lane];
+            }
           }
-        }
-        if (BASE) {
-          for (int ww = 0; ww < kConsumerWarps; ++ww) {
-            const uint64_t k = red[(buf * kConsumerWarps + ww) * kRedPerWarp + 2 * S];
-            v2 = k > v2 ? k : v2;
+          if (BASE) {
+            for (int ww = warp; ww < warp + gw; ++ww) {
+              const uint64_t k = red[(buf * kConsumerWarps + ww) * kRedPerWarp + 2 * S];
+              v2 = k > v2 ? k : v2;
+            }
           }
+          if constexpr (MODE == 0) finalize_frontier(p, S, t, v0, lane, acc);
+          else if constexpr (BASE) finalize_base(p, S, t, v0, v1, v2, lane, bacc);
+          else finalize_gain(p, S, t, v0, static_cast<int64_t>(v1), lane, acc);
         }
-        if constexpr (MODE == 0) finalize_frontier(p, S, t, v0, lane, acc);
-        else if constexpr (BASE) finalize_base(p, S, t, v0, v1, v2, lane, bacc);
-        else finalize_gain(p, S, t, v0, static_cast<int64_t>(v1), lane, acc);
+        buf ^= 1;
       }
-      buf ^= 1;
-    }
+    };
+    if (p.groups == 4) consume(std::integral_constant<int, 4>{});
+    else if (p.groups == 2) consume(std::integral_constant<int, 2>{});
+    else consume(std::integral_constant<int, 1>{});
   }
 
-  if (BASE && (p.regime == 0 || warp == 0)) flush_base(p, S, bacc, lane);
-  if (!BASE && p.X && (p.regime == 0 || warp == 0)) flush_window(p, S, acc, lane);
+  const bool leader = p.regime == 0 || warp % (kConsumerWarps / p.groups) == 0;  // holds window accumulators
+  if (BASE && leader) flush_base(p, S, bacc, lane);
+  if (!BASE && p.X && leader) flush_window(p, S, acc, lane);
   if (GAIN && p.quality) qual_window(p, qa, -2, lane);
   const uint32_t bits = range_bits(__reduce_or_sync(kFull, dor), __reduce_or_sync(kFull, tor)) |
                         (*abort ? SF_ST_TIMEOUT : 0u);
@@ -1014,6 +1065,12 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
     p.m_by_tma = (j.gain && p.regime == 1) ? 1 : 0;
     p.nst = p.regime == 0 ? kR0Stages : p.m_by_tma ? kR1GainStages : kR1Stages;
     p.stage_bytes = p.regime == 0 ? kR0StageBytes : p.m_by_tma ? kR1GainStageBytes : kR1StageBytes;
+    // Small steps in regime 1: groups of warps take steps in turn, so that
+    // several steps' reductions are in flight.  Each group owns nst / groups
+    // ring stages: a stage is refilled only after its own group has consumed
+    // it, so no wait can pass a phase early.
+    p.groups = 1;
+    if (p.regime == 1 && p.nst >= 4) p.groups = p.tiles_per_step == 1 && step_rows <= 128 ? 4 : p.tiles_per_step <= 2 ? 2 : 1;
     if (p.m_by_tma) {
       const int64_t nW = (j.T + j.W - 1) / j.W;
       if (nW * step_rows > int64_t(0x7fffffff) || encode(&map_m, j.m, nW * step_rows) != CUDA_SUCCESS)
