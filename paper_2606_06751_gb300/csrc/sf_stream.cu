@@ -17,7 +17,9 @@
 // prefix and per-boundary maxima in registers, and reduce across ranks with
 // warp redux plus one shared-memory exchange.  Small steps (<= 12 KB) are
 // handled by one warp per tile of whole steps, each warp owning two ring
-// stages; large steps one step per CTA spread over several tiles.
+// stages; larger steps by one warp group per step, spread over one or more
+// tiles, with two or four groups taking steps of one or two tiles in turn
+// (each group owning its ring stages) and all eight warps on larger steps.
 //
 // Generic path (any other S <= 32 or R): one CTA per step range with plain
 // global loads.  Both paths share the per-step epilogues.
