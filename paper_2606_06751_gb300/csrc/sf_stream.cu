@@ -618,7 +618,47 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
       const bool have = mbar_wait_bounded(&full[st], ph, abort);
       const unsigned char* tile = ring + size_t(st) * kR0StageBytes;
       const int nsteps = static_cast<int>(min(int64_t(p.K), n_local - j * p.K));
-      for (int kk = 0; kk < nsteps; ++kk) {
+      int kk0 = 0;
+      if constexpr (MODE == 0 && S <= 8) {
+        // frontier steps in pairs: two independent reduction chains per warp
+        constexpr int UP = S <= 4 ? 2 : 1;  // rank rows of each step in flight per lane
+        for (; kk0 + 1 < nsteps; kk0 += 2) {
+          const int64_t t = t_begin + j * p.K + kk0;
+          FrontierRows<S> ra, rb;
+          ra.init();
+          rb.init();
+          if (have) {
+            for (int r0 = lane; r0 < R; r0 += 32 * UP) {
+              int64_t va[UP][S], vb[UP][S];
+#pragma unroll
+              for (int u = 0; u < UP; ++u)
+                if (r0 + 32 * u < R) {
+                  load_row<S, kSwz>(tile, kk0 * R + r0 + 32 * u, va[u]);
+                  load_row<S, kSwz>(tile, (kk0 + 1) * R + r0 + 32 * u, vb[u]);
+                }
+#pragma unroll
+              for (int u = 0; u < UP; ++u)
+                if (r0 + 32 * u < R) {
+                  ra.row(va[u], r0 + 32 * u, dor, tor);
+                  rb.row(vb[u], r0 + 32 * u, dor, tor);
+                }
+            }
+          }
+          uint64_t ka = 0, kb = 0;
+#pragma unroll
+          for (int s = 0; s < S; ++s) {
+            const uint64_t ma = warp_max_u64(ra.key(s));
+            const uint64_t mb = warp_max_u64(rb.key(s));
+            if (lane == s) {
+              ka = ma;
+              kb = mb;
+            }
+          }
+          finalize_frontier(p, S, t, ka, lane, acc);
+          finalize_frontier(p, S, t + 1, kb, lane, acc);
+        }
+      }
+      for (int kk = kk0; kk < nsteps; ++kk) {
         const int64_t t = t_begin + j * p.K + kk;
         const int64_t w = GAIN ? t / p.W : 0;
         if (GAIN && p.quality) qual_window(p, qa, w, lane);
