@@ -57,8 +57,12 @@ SHAPES = [
     (9, 520, 12), (6, 1000, 14), (4, 512, 8), (3, 65536, 2),
 ]
 
+# one-step-per-CTA shapes whose steps are one or two tiles go to two or four
+# warp groups in turn, each group flushing its own window sums
+GROUPED = [(9, 520, 12), (6, 1000, 14), (4, 512, 8), (3000, 512, 4), (700, 768, 6), (301, 2048, 2)]
 
-@pytest.mark.parametrize("T,R,S", SHAPES)
+
+@pytest.mark.parametrize("T,R,S", SHAPES + GROUPED[4:])
 @pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal"])
 def test_frontier_parity(sf, T, R, S, kind):
     d_np = make(T, R, S, T * 131 + R * 7 + S, kind)
@@ -105,7 +109,7 @@ def test_long_ranges_reuse_ring(sf, T, R, S):
     assert np.array_equal(host(ev.Y)[:2], O.direct_gain(d_np[:2 * W], W, m2))
 
 
-@pytest.mark.parametrize("T,R,S", SHAPES[:4] + SHAPES[5:9] + SHAPES[14:18])
+@pytest.mark.parametrize("T,R,S", SHAPES[:4] + SHAPES[5:9] + SHAPES[14:18] + GROUPED)
 @pytest.mark.parametrize("t0,W", [(0, 7), (13, 10), (0, 1000)])
 def test_window_aggregate_parity(sf, T, R, S, t0, W):
     d_np = make(T, R, S, T + R + S + t0, "ties" if R < 100 else "lognormal")
@@ -304,7 +308,7 @@ def test_bounded_wait_times_out_cleanly(sf):
     assert np.array_equal(host(f.a), O.frontier(host(d)).a)
 
 
-@pytest.mark.parametrize("T,R,S", SHAPES[:4] + SHAPES[5:9] + SHAPES[14:18] + [(3000, 512, 4), (200000, 8, 6)])
+@pytest.mark.parametrize("T,R,S", SHAPES[:4] + SHAPES[5:9] + SHAPES[14:18] + GROUPED + [(200000, 8, 6)])
 @pytest.mark.parametrize("t0,W", [(0, 7), (13, 100)])
 def test_baselines_parity(sf, T, R, S, t0, W):
     """Per-stage max, sum (128-bit), slowest-rank breakdown and rank-0 total
