@@ -41,7 +41,7 @@ constexpr int kSelThreads = 128;
 constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kSelPerSM = 1536 / kSelThreads;  // resident select CTAs per SM
 constexpr int kSelCand = 2048;  // candidate keys a column may keep after the second pass
-constexpr size_t kRkChunkTarget = size_t(40) << 20;  // scratch of one chunk buffer; two fit L2
+constexpr size_t kRkChunkTarget = size_t(52) << 20;  // scratch of one chunk buffer; two fit L2 (52 MB: 207 steps of 8192 x 8, one select wave)
 
 struct RankParams {
   const int64_t* d;
