@@ -562,6 +562,70 @@ def test_stage_group_sum():
     assert (y[:, 0] == w.X[:, 0::2].sum(axis=1)).all() and (y.sum(axis=1) == w.D).all()
 
 
+def _lower_median_by_counting(col):
+    """The smallest value v of the column with #{x <= v} >= ceil(n/2): for an
+    even n this is the lower of the two middle values, for an odd n the median."""
+    n = len(col)
+    return min(v for v in col if sum(1 for x in col if x <= v) >= (n + 1) // 2)
+
+
+@pytest.mark.parametrize("R", [2, 4, 8, 64])
+def test_lag_even_ranks_take_the_lower_median(R):
+    """Sec. 4 lag L = max_r P - median_r P with an even number of ranks: the
+    median is the lower of the two middle prefixes (the reading that keeps the
+    lag an exact integer).  Checked against numpy's 'lower' percentile and a
+    brute-force count, on data with many ties."""
+    rng = np.random.default_rng(800 + R)
+    T, S = 9, 4
+    d = rand_d(rng, T, R, S, hi=6, zero_frac=0.3)           # few distinct values: ties
+    g = O.rank_lag(d)
+    P = np.cumsum(d, axis=2)
+    F = P.max(axis=1)
+    lower = np.percentile(P, 50, axis=1, method="lower").astype(np.int64)
+    assert (g.L == F - lower).all()
+    for t in range(T):
+        for s in range(S):
+            assert g.L[t, s] == F[t, s] - _lower_median_by_counting(list(P[t, :, s]))
+    second = np.sort(P, axis=1)[:, -2, :]
+    assert (g.G == F - second).all()
+    # the upper middle value would give a different lag somewhere on this data
+    upper = np.sort(P, axis=1)[:, R // 2, :]
+    assert (lower != upper).any()
+
+
+def test_lag_and_spread_four_rank_fixture():
+    """Hand fixture for the even-R reading: one step, one stage, four ranks
+    with durations (= prefixes) 5, 9, 1, 2.  Sorted 1 2 5 9: the lower middle
+    value is 2, so L = 9 - 2 = 7 (the upper middle would give 4, the mean of
+    the two 5.5); the gap to the second largest is 9 - 5 = 4; the raw spread
+    of the window is the same 7."""
+    d = np.array([[[5], [9], [1], [2]]], np.int64)
+    g = O.rank_lag(d)
+    assert g.L.tolist() == [[7]] and g.G.tolist() == [[4]] and g.dL.tolist() == [[7]]
+    assert O.raw_spread(d, 1).tolist() == [[7]]
+    # two stages: prefixes (5,8) (9,9) (1,11) (2,2) -> stage 1 column 8 9 11 2,
+    # sorted 2 8 9 11, lower middle 8: L = 11 - 8 = 3, delta-lag 3 - 7 = -4
+    d2 = np.array([[[5, 3], [9, 0], [1, 10], [2, 0]]], np.int64)
+    g2 = O.rank_lag(d2)
+    assert g2.L.tolist() == [[7, 3]] and g2.dL.tolist() == [[7, -4]] and g2.G.tolist() == [[4, 2]]
+    # spread of the durations: stage 0 as above (7); stage 1 column 3 0 10 0,
+    # sorted 0 0 3 10, lower middle 0: 10 - 0 = 10
+    assert O.raw_spread(d2, 1).tolist() == [[7, 10]]
+
+
+@pytest.mark.parametrize("R", [2, 8, 64])
+def test_raw_spread_even_ranks_take_the_lower_median(R):
+    rng = np.random.default_rng(900 + R)
+    T, S, W = 14, 3, 5
+    d = rand_d(rng, T, R, S, hi=5, zero_frac=0.2)
+    sp = O.raw_spread(d, W)
+    per_step = d.max(axis=1) - np.percentile(d, 50, axis=1, method="lower").astype(np.int64)
+    for w in range(sp.shape[0]):
+        assert (sp[w] == per_step[w * W:(w + 1) * W].sum(axis=0)).all()
+    t, s = 3, 1
+    assert per_step[t, s] == d[t, :, s].max() - _lower_median_by_counting(list(d[t, :, s]))
+
+
 def test_lag_windows():
     # window sums of the per-step evidence; a stall Delta on one of otherwise
     # identical ranks at step t contributes Delta to every stage from the
