@@ -394,7 +394,11 @@ size_t sf_stream_gathered_staging_size(int64_t T, int64_t R, int64_t S, int64_t 
  *
  * Set-up: the first call on each device looks up the array's device address
  * (cudaGetSymbolAddress) with that device current, and caches it; make that
- * first call before any stream capture.
+ * first call before any stream capture.  The cached address belongs to the
+ * device's current primary context: after cudaDeviceReset (or any other
+ * reset of that context) the module is loaded afresh and the array may move,
+ * so do not call this entry point again in a process that has reset the
+ * device.
  *
  * Sharing: all calls on a device use the same array, and it keeps whatever
  * the last call left there.  Each call zeroes the parts it accumulates into,

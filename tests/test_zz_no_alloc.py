@@ -4,9 +4,10 @@ the device memory, where a cudaMalloc from the hook could stall the step it
 measures).  Its intermediates live in the library's static device scratch.
 
 Both entry points are called through the C ABI on the same inputs; the
-no-allocation one must agree with the workspace one on two calls in a row
-(the second on different data, so stale scratch from the first call would
-show), and must refuse a problem larger than its static scratch.  This file
+no-allocation one must agree with the workspace one and with the CPU oracle
+on two calls in a row (the second on different data, so stale scratch from
+the first call would show), and must refuse a problem larger than its static
+scratch.  This file
 is collected last so a failure here does not hide the rest of the suite."""
 import ctypes
 
@@ -14,6 +15,7 @@ import numpy as np
 import pytest
 import torch
 
+from oracle import oracle as O
 from synth import workloads as wl
 
 pytestmark = pytest.mark.gpu
@@ -67,6 +69,11 @@ def _same(a, b):
             assert np.array_equal(x, y), i
 
 
+def _oracle(d_np, W, missing):
+    o = O.label_windows(d_np, W, missing=missing)
+    return [o.labels, o.route_mask, o.amb_mask, o.share, o.gain, o.X, o.Y, o.D]
+
+
 def test_noalloc_matches_workspace_entry_point_twice(sf):
     first = wl.fsdp1024(steps=1000).generate()          # 2 windows of 500 steps
     second = wl.accum8192(steps=120, seed=3).generate()  # different shape and data
@@ -77,6 +84,10 @@ def test_noalloc_matches_workspace_entry_point_twice(sf):
         ref = _call(sf, d, W, use_static=False, missing=missing)
         got = _call(sf, d, W, use_static=True, missing=missing)
         _same(got, ref)
+        # the CPU oracle on the same input: integer outputs bit-exact, the
+        # fp64 shares and gains within 1e-12 relative
+        orc = _oracle(d_np, W, np.zeros(nW, np.int32))
+        _same([g.astype(o.dtype) for g, o in zip(got, orc)], orc)
         # a second call in a row on the same data sees the scratch the first one left
         _same(_call(sf, d, W, use_static=True, missing=missing), ref)
 
