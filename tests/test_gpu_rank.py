@@ -80,6 +80,50 @@ def test_rank_lag_parity(sf, T, R, S, kind):
     assert np.array_equal(host(g.G), o.G)
 
 
+def make_stream(T, R, S, seed, kind):
+    """Inputs for the streaming pass, where a CTA walks many consecutive steps
+    and predicts each step's median from the last: smooth steps, steps whose
+    level jumps up and down (the prediction misses on both sides), heavy ties
+    (candidate segments overflow), rare wide values (the 64-bit fallback) and
+    values at the 32-bit limits of the main pass."""
+    rng = np.random.default_rng(seed)
+    if kind in ("lognormal", "mixed", "cluster", "boundary", "ties"):
+        return make(T, R, S, seed, kind)
+    med = rng.uniform(1e6, 5e7, size=S)
+    d = np.rint(med * np.exp(0.1 * rng.standard_normal((T, R, S)))).astype(np.int64)
+    if kind == "jumps":      # every step's level drawn anew: 0.2x .. 5x
+        d = np.rint(d * np.exp(rng.uniform(-1.6, 1.6, size=(T, 1, 1)))).astype(np.int64)
+    if kind == "drift":      # a slow trend with occasional 3x steps
+        f = np.exp(np.cumsum(rng.normal(0, 0.02, size=T)))
+        f[rng.random(T) < 0.05] *= 3
+        d = np.rint(d * f[:, None, None]).astype(np.int64)
+    if kind == "narrow":     # the spread collapses for some steps: few distinct values
+        sel = rng.random(T) < 0.3
+        d[sel] = (d[sel] // 100000) * 100000
+    return d
+
+
+@pytest.mark.parametrize("T,R,S", [(3000, 1024, 8), (2000, 2048, 4), (1500, 1024, 16), (700, 4096, 8)])
+@pytest.mark.parametrize("kind", ["lognormal", "jumps", "drift", "narrow", "mixed", "cluster", "ties", "boundary"])
+def test_rank_lag_streaming_many_steps(sf, T, R, S, kind):
+    """Many steps per CTA (the grid holds two CTAs per SM), so most steps are
+    resolved from the predicted bracket and the rest by the exact fallback."""
+    d_np = make_stream(T, R, S, T + R + S, kind)
+    o = O.rank_lag(d_np)
+    st = sf.new_status("cuda")
+    g = sf.sf_rank_lag(dev(d_np), status=st)
+    sp = sf.sf_raw_spread(dev(d_np), 100, t0=7, status=st)
+    lw = sf.sf_rank_lag_windows(dev(d_np), 100, t0=7, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert np.array_equal(host(g.L), o.L)
+    assert np.array_equal(host(g.dL), o.dL)
+    assert np.array_equal(host(g.G), o.G)
+    assert np.array_equal(host(sp), O.raw_spread(d_np, 100, 7))
+    LW, GW = O.rank_lag_windows(d_np, 100, t0=7)
+    assert np.array_equal(host(lw[0]), LW) and np.array_equal(host(lw[1]), GW)
+
+
 def test_rank_lag_optional_outputs(sf):
     d_np = make(40, 33, 6, 5, "lognormal")
     o = O.rank_lag(d_np)
