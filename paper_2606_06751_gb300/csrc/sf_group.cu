@@ -107,10 +107,15 @@ __global__ void __launch_bounds__(kGrThreads) group_window_kernel(const GroupPar
   const int64_t t_begin = q * b + (b < rr ? b : rr), t_end = t_begin + q + (b < rr ? 1 : 0);
   uint32_t dor = 0, tor = 0, bad_group = 0;
   int64_t cur_w = -1;
+  int64_t w = 0, w_lo = 0, w_hi = 0;  // steps [w_lo, w_hi) form window w: one division per window
 
   for (int i = tid; i < GS + G; i += kGrThreads) accX[i] = 0;  // accX and accD are contiguous
   for (int64_t t = t_begin; t < t_end; ++t) {
-    const int64_t w = (p.t0 + t) / p.W - p.w_first;
+    if (t < w_lo || t >= w_hi) {
+      w = (p.t0 + t) / p.W - p.w_first;
+      w_lo = (w + p.w_first) * p.W - p.t0;
+      w_hi = w_lo + p.W;
+    }
     for (int i = tid; i < GS; i += kGrThreads) Fk[i] = 0;
     if (w != cur_w && cur_w >= 0) {
       // the window changed: add the finished window's sums to global memory

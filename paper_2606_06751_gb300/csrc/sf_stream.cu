@@ -98,11 +98,27 @@ __device__ __forceinline__ uint32_t hi32(int64_t v) {
 }
 
 // --------------------------------------------------------------------------
+// Window index of step t, (t0 + t) / W - w_first, recomputed (one 64-bit
+// division) only when t leaves the last window seen: the steps a thread
+// visits increase, so that happens once per window rather than once per step.
+struct WinTrack {
+  int64_t lo = 0, hi = 0, w = 0;  // steps [lo, hi) belong to window w
+  __device__ __forceinline__ int64_t at(int64_t t, int64_t t0, int64_t W, int64_t w_first) {
+    if (t < lo || t >= hi) {
+      w = (t0 + t) / W - w_first;
+      lo = (w + w_first) * W - t0;
+      hi = lo + W;
+    }
+    return w;
+  }
+};
+
 // Window accumulators held by the warp that finalizes steps: lane s keeps the
 // stage-s numerators, every lane the denominator.
 struct WinAcc {
   int64_t cur = -1;
   int64_t x = 0, y = 0, dsum = 0;
+  WinTrack wt;
 };
 
 __device__ __forceinline__ void flush_window(const Params& p, int S, WinAcc& acc, int lane) {
@@ -138,7 +154,7 @@ __device__ __forceinline__ void finalize_frontier(const Params& p, int S, int64_
   }
   if (lane == 0 && p.mk) p.mk[t] = mk;
   if (p.X) {
-    const int64_t w = (p.t0 + t) / p.W - p.w_first;
+    const int64_t w = acc.wt.at(t, p.t0, p.W, p.w_first);
     if (w != acc.cur) {
       flush_window(p, S, acc, lane);
       acc.cur = w;
@@ -181,7 +197,7 @@ __device__ __forceinline__ void finalize_gain(const Params& p, int S, int64_t t,
   const bool conf = FS > 0 && static_cast<__int128>(amax - second) * p.eta_den >=
                                   static_cast<__int128>(p.eta_num) * FS;
   if (lane == 0) p.step_lead[t] = static_cast<uint8_t>(best | (conf ? SF_STEP_CONFIDENT : 0u));
-  const int64_t w = t / p.W;
+  const int64_t w = acc.wt.at(t, 0, p.W, 0);
   if (w != acc.cur) {
     flush_window(p, S, acc, lane);
     acc.cur = w;
@@ -202,6 +218,7 @@ struct BaseAcc {
   int64_t cur = -1;
   int64_t m = 0, slow = 0, r0 = 0;
   unsigned __int128 sum = 0;
+  WinTrack wt;
 };
 
 __device__ __forceinline__ void flush_base(const Params& p, int S, BaseAcc& acc, int lane) {
@@ -223,7 +240,7 @@ __device__ __forceinline__ void flush_base(const Params& p, int S, BaseAcc& acc,
 // back from d (the step was just streamed, so these hit L2).
 __device__ __forceinline__ void finalize_base(const Params& p, int S, int64_t t, uint64_t mx, uint64_t sm,
                                               uint64_t slowkey, int lane, BaseAcc& acc) {
-  const int64_t w = (p.t0 + t) / p.W - p.w_first;
+  const int64_t w = acc.wt.at(t, p.t0, p.W, p.w_first);
   if (w != acc.cur) {
     flush_base(p, S, acc, lane);
     acc.cur = w;
@@ -527,6 +544,7 @@ __device__ void produce(const CUtensorMap* map, const CUtensorMap* map_m, const 
     if (p.m_by_tma) tma_load_2d(dst + p.stage_bytes / 2, map_m, 0, static_cast<int32_t>(mrow), &full[st]);
     ++j;
   };
+  WinTrack mw;  // window of the medians streamed beside d (evidence pass)
   if (p.regime == 0) {
     for (int64_t t = t_begin; t < t_end && ok; t += p.K) {
       uint32_t st, ph;
@@ -539,7 +557,7 @@ __device__ void produce(const CUtensorMap* map, const CUtensorMap* map_m, const 
     for (int64_t t = t_begin; t < t_end && ok; ++t)
       for (int k = 0; k < p.tiles_per_step && ok; ++k) {
         const int64_t r0 = min(int64_t(k) * p.box_rows, p.step_rows - p.box_rows);
-        issue(t * p.step_rows + r0, (t / p.W) * p.step_rows + r0, rg.slot, rg.ph);
+        issue(t * p.step_rows + r0, mw.at(t, 0, p.W, 0) * p.step_rows + r0, rg.slot, rg.ph);
         rg.advance(nst);
       }
   } else {
@@ -551,7 +569,7 @@ __device__ void produce(const CUtensorMap* map, const CUtensorMap* map_m, const 
       uint32_t slot = (walk >> sh) & 7u, ph = (walk >> (sh + 3)) & 1u;
       for (int k = 0; k < p.tiles_per_step && ok; ++k) {
         const int64_t r0 = min(int64_t(k) * p.box_rows, p.step_rows - p.box_rows);
-        issue(t * p.step_rows + r0, (t / p.W) * p.step_rows + r0, g + G * slot, ph);
+        issue(t * p.step_rows + r0, mw.at(t, 0, p.W, 0) * p.step_rows + r0, g + G * slot, ph);
         if (++slot == spg) {
           slot = 0;
           ph ^= 1u;
@@ -605,6 +623,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
   uint32_t dor = 0, tor = 0;  // OR of duration / rank-total high words
   WinAcc acc;
   QualAcc qa;
+  WinTrack qt;  // window of the step a warp is on (evidence pass)
   BaseAcc bacc;
   const int R = static_cast<int>(p.R);
 
@@ -660,7 +679,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
       }
       for (int kk = kk0; kk < nsteps; ++kk) {
         const int64_t t = t_begin + j * p.K + kk;
-        const int64_t w = GAIN ? t / p.W : 0;
+        const int64_t w = GAIN ? qt.at(t, 0, p.W, 0) : 0;
         if (GAIN && p.quality) qual_window(p, qa, w, lane);
         const int q0 = kk * R;
         if constexpr (MODE == 0) {
@@ -753,7 +772,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
       GroupRing gring;
       int buf = 0;
       for (int64_t t = t_begin + g; t < t_end; t += NG) {
-        const int64_t w = GAIN ? t / p.W : 0;
+        const int64_t w = GAIN ? qt.at(t, 0, p.W, 0) : 0;
         if (GAIN && p.quality) qual_window(p, qa, w, lane);
         [[maybe_unused]] FrontierRows<S> fr;
         [[maybe_unused]] GainRows<S> gr;
@@ -897,9 +916,10 @@ __global__ void __launch_bounds__(kGenThreads)
   uint32_t dor = 0, tor = 0;
   WinAcc acc;
   QualAcc qa;
+  WinTrack qt;  // window of the step a warp is on (evidence pass)
   BaseAcc bacc;
   for (int64_t t = t_begin; t < t_end; ++t) {
-    const int64_t w = GAIN ? t / p.W : 0;
+    const int64_t w = GAIN ? qt.at(t, 0, p.W, 0) : 0;
     if (GAIN && p.quality) qual_window(p, qa, w, lane);
     int64_t b0[32], b1[32];
     int32_t br[32];
