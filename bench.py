@@ -370,6 +370,16 @@ def run_ours(args):
                              args.warmup, ws, device, True) / args.steps
     del g_dev
 
+    # every other configuration (the three smaller workloads and the twelve
+    # 1 GiB sweep shapes): frontier and aggregation passes and the whole step
+    # on the GPU, the oracle on a bounded sample single-threaded and on all cores
+    configs = None
+    if ws == 1 and not args.no_configs:
+        from oracle import oracle as O
+        O.build_lib()
+        configs = [measure_config(n, sf, device, peak, 5, 3, args.seed, oracle=O)
+                   for n in CONFIG_NAMES if n != w.name]
+
     # end to end through the host-memory entry point: every step streams the
     # pinned host tensor to the GPU in 2000-step chunks (copies overlapping the
     # previous chunk's compute) and reads the per-window results back
@@ -388,7 +398,20 @@ def run_ours(args):
         for hb, o in zip(host_outs, outs):
             hb.copy_(o, non_blocking=True)
 
-    e2e_steps = max(3, args.steps // 2)
+    # the host link's own rate for the same bytes: plain pinned copies of the
+    # same chunks into one device buffer, timed before and after the e2e legs
+    # (the link is shared with the machine's other tenants and drifts)
+    link_buf = torch.empty((chunk, w.R, w.S), dtype=torch.int64, device=device)
+
+    def link_pass():
+        for c0 in range(0, w.T, chunk):
+            n = min(chunk, w.T - c0)
+            link_buf[:n].copy_(host[c0:c0 + n], non_blocking=True)
+
+    link_steps = 5
+    link_before = w.nbytes * ws * link_steps / timed_loop(link_pass, link_steps, 3, ws, device, True) / 1e9
+
+    e2e_steps = max(20, args.steps)
     e2e_secs = timed_loop(e2e_step, e2e_steps, args.warmup, ws, device, True)
     e2e_value = records * ws * e2e_steps / e2e_secs
 
@@ -405,7 +428,21 @@ def run_ours(args):
             hb.copy_(o, non_blocking=True)
 
     e2e_g_secs = timed_loop(e2e_gathered_step, e2e_steps, args.warmup, ws, device, True)
-    del gbufs, g_host
+    link_after = w.nbytes * ws * link_steps / timed_loop(link_pass, link_steps, 3, ws, device, True) / 1e9
+    link_gbs = (link_before + link_after) / 2
+    # the gathered leg reads another pinned buffer, whose pages can sit
+    # elsewhere in host memory: its own link rate, measured the same way
+    g_flat = g_host.view(-1)
+    link_flat = link_buf.view(-1)
+
+    def link_pass_gathered():
+        step_words = w.R * w.S
+        for c0 in range(0, w.T, chunk):
+            n = min(chunk, w.T - c0) * step_words
+            link_flat[:n].copy_(g_flat[c0 * step_words:c0 * step_words + n], non_blocking=True)
+
+    link_g_gbs = w.nbytes * ws * link_steps / timed_loop(link_pass_gathered, link_steps, 3, ws, device, True) / 1e9
+    del gbufs, g_host, g_flat, link_flat, link_buf
     if int(pipe.status.item()) != 0:
         raise RuntimeError("device status set during the end-to-end loop")
 
@@ -419,11 +456,7 @@ def run_ours(args):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
-        "config": {"workload": f"{w.name}: {w.R} ranks x {w.S} stages x {w.T} steps int64 ns "
-                               f"({w.nbytes / 1e9:.2f} GB), windows of {w.W}, top-{w.k}, labels",
-                   "R": w.R, "S": w.S, "T": w.T, "W": w.W, "k": w.k, "seed": args.seed,
-                   "l2": f"input {w.nbytes / 1e9:.1f} GB > 129 MB L2 on every pass; no flush",
-                   "parallelism": "replicas" if ws > 1 else "single"},
+        "config": workload_config(w, args, ws),
         "step_gbs": sum(algo[n] for n in pipe.names) / (secs / args.steps) / 1e9,
         "roofline": {"kernel": dominant, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
                      "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
@@ -448,12 +481,20 @@ def run_ours(args):
                         "gbs": round(2 * w.nbytes / ingest_secs / 1e9, 1),
                         "frac": round(2 * w.nbytes / ingest_secs / 1e9 / peak, 4)},
         "e2e_gathered": {"value": records * ws * e2e_steps / e2e_g_secs, "unit": UNIT,
-                         "entry": "sf_stream_gathered_windows", "h2d_bytes_per_step": w.nbytes},
+                         "entry": "sf_stream_gathered_windows", "h2d_bytes_per_step": w.nbytes,
+                         "steps": e2e_steps, "h2d_gbs": round(w.nbytes * ws * e2e_steps / e2e_g_secs / 1e9, 1),
+                         "link_gbs": round(link_g_gbs, 1),
+                         "frac_of_link": round(w.nbytes * ws * e2e_steps / e2e_g_secs / 1e9 / link_g_gbs, 3)},
         "gpu_launches": int(launches * args.steps // (args.steps + args.warmup)),
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": w.nbytes, "d2h_bytes_per_step": d2h,
-                "entry": "sf_stream_windows", "chunk_steps": chunk},
+                "entry": "sf_stream_windows", "chunk_steps": chunk, "steps": e2e_steps,
+                "h2d_gbs": round(w.nbytes * ws * e2e_steps / e2e_secs / 1e9, 1),
+                "link_gbs": round(link_gbs, 1), "link_gbs_before_after": [round(link_before, 1), round(link_after, 1)],
+                "frac_of_link": round(w.nbytes * ws * e2e_steps / e2e_secs / 1e9 / link_gbs, 3)},
         "clocks": clk.summary(),
     }
+    if configs is not None:
+        line["configs"] = configs
     if ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, args.cpu_sample_windows)
     return line
@@ -468,50 +509,165 @@ def oracle_step(O, w: wl.Workload, d_np: np.ndarray):
     O.label_windows(d_np, w.W)
 
 
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo), for the report."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith(("model name", "cpu part")):
+                return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return "unknown"
+
+
+def oracle_rate(O, w: wl.Workload, n: int, threads: int) -> dict:
+    """The oracle on `threads` disjoint slices of n steps each (slice i: steps
+    [i n, (i+1) n) of the workload, windows of min(W, n) steps), one host
+    thread per slice (the C oracle releases the GIL).  Returns records/s over
+    the wall time of all slices together."""
+    from concurrent.futures import ThreadPoolExecutor
+    n = max(1, min(n, w.T // threads))
+    wn = min(w.W, n)
+    slices = [w.generate(t0=i * n, nsteps=n) for i in range(threads)]
+    sw = wl.Workload(**{**w.__dict__, "T": n, "W": wn})
+    t0 = time.perf_counter()
+    if threads == 1:
+        oracle_step(O, sw, slices[0])
+    else:
+        with ThreadPoolExecutor(threads) as ex:
+            list(ex.map(lambda x: oracle_step(O, sw, x), slices))
+    secs = time.perf_counter() - t0
+    rec = threads * n * w.R * w.S
+    return {"value": rec / secs, "unit": UNIT, "cores": threads, "kind": "oracle", "secs": round(secs, 2),
+            "sample": f"{threads} x {n} steps of {w.name} (windows of {wn}): {rec} records"}
+
+
 def cpu_baseline(w: wl.Workload, n_windows: int):
+    """The CPU oracle on the host's cores: single-threaded on the first
+    n_windows windows, and on all cores over disjoint window ranges."""
     from oracle import oracle as O
     n = min(w.T, n_windows * w.W)
-    d_np = w.generate(t0=0, nsteps=n)
-    t0 = time.perf_counter()
-    oracle_step(O, w, d_np)
-    secs = time.perf_counter() - t0
-    rec = n * w.R * w.S
-    return {"value": rec / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"first {n} steps ({n // w.W} windows) of {w.name}: {rec} records, "
-                      f"{secs:.1f} s single-threaded C oracle (frontier/windows, top-k, medians, gains, gates)"}
+    one = oracle_rate(O, w, n, 1)
+    cores = os.cpu_count() or 1
+    per = max(w.W, (w.T // cores) // w.W * w.W)  # whole windows per thread, all of T at most
+    threads = max(1, min(cores, w.T // per))
+    allc = oracle_rate(O, w, per, threads)
+    return {"value": one["value"], "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"first {n} steps ({n // w.W} windows) of {w.name}: {n * w.R * w.S} records, "
+                      f"{one['secs']} s single-threaded C oracle (frontier/windows, top-k, medians, gains, gates)",
+            "all_cores": {"value": allc["value"], "cores": allc["cores"], "sample": allc["sample"],
+                          "secs": allc["secs"]},
+            "host_cpus": cores, "cpu_model": cpu_model()}
+
+
+def workload_config(w: wl.Workload, args, ws: int) -> dict:
+    """The `config` object of the JSON line (the same for both arms)."""
+    return {"workload": f"{w.name}: {w.R} ranks x {w.S} stages x {w.T} steps int64 ns "
+                        f"({w.nbytes / 1e9:.2f} GB), windows of {w.W}, top-{w.k}, labels",
+            "R": w.R, "S": w.S, "T": w.T, "W": w.W, "k": w.k, "seed": args.seed,
+            "l2": f"input {w.nbytes / 1e9:.1f} GB > 129 MB L2 on every pass; no flush",
+            "parallelism": "replicas" if ws > 1 else "single"}
 
 
 def run_reference(args):
+    """The CPU oracle as the reference arm: each step runs the whole hot path
+    (frontier and windows, top-k, medians, gains, gates) on whole windows of
+    the workload, one window per host core over disjoint windows (the C
+    oracle releases the GIL), so a step does the same per-window work as a
+    GPU step on a bounded sample of its windows."""
+    from concurrent.futures import ThreadPoolExecutor
     ws, rank, _ = dist_env()
     if rank != 0:
         return None
     from oracle import oracle as O
     O.build_lib()
     w = wl.by_name(args.workload, seed=args.seed, steps=args.steps_override)
-    n = min(w.T, args.ref_sample_steps)
-    d_np = w.generate(t0=0, nsteps=n)
-    ww = wl.Workload(**{**w.__dict__, "T": n})
+    cores = os.cpu_count() or 1
+    nwin = max(1, min(cores, w.T // w.W))
+    slices = [w.generate(t0=i * w.W, nsteps=min(w.W, w.T - i * w.W)) for i in range(nwin)]
+    sw = wl.Workload(**{**w.__dict__, "T": w.W})
+
+    def step():
+        with ThreadPoolExecutor(nwin) as ex:
+            list(ex.map(lambda x: oracle_step(O, sw, x), slices))
+
     for _ in range(args.warmup):
-        oracle_step(O, ww, d_np)
+        step()
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        oracle_step(O, ww, d_np)
+        step()
     secs = time.perf_counter() - t0
-    rec = n * w.R * w.S
+    rec = sum(x.shape[0] for x in slices) * w.R * w.S
     value = rec * args.steps / secs
-    sample = (f"each step: first {n} steps of {w.name} ({rec} records; a window shorter than "
-              f"{w.W} steps), single-threaded C oracle")
+    sample = (f"each step: windows 0..{nwin - 1} of {w.name} ({nwin} whole windows of {w.W} steps, "
+              f"{rec} records), one per host thread, C oracle")
     return {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
-        "data": "synthetic",
-        "config": {"workload": f"{w.name}: {w.R} ranks x {w.S} stages x {w.T} steps int64 ns, "
-                               f"windows of {w.W}, top-{w.k}, labels", "R": w.R, "S": w.S, "T": w.T,
-                   "W": w.W, "k": w.k, "seed": args.seed, "sample_steps": n},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "data": "synthetic", "config": workload_config(w, args, ws),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": nwin, "kind": "oracle", "sample": sample,
+                         "host_cpus": cores, "cpu_model": cpu_model()},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
+
+
+CONFIG_NAMES = ["tiny", "ddp128", "fsdp1024", "accum8192"] + [f"sweep_R{R}_S{S}" for R in wl.SWEEP_R
+                                                                for S in wl.SWEEP_S]
+ORACLE_SAMPLE_RECORDS = 4_000_000  # per oracle thread, per configuration
+
+
+def measure_config(name: str, sf, device, peak: float, steps: int, warmup: int, seed: int, oracle=None) -> dict:
+    """Frontier pass (sf_frontier), aggregation pass (sf_window_aggregate) and
+    whole step on one synthetic configuration, device-resident, CUDA events;
+    with `oracle`, the CPU oracle on a bounded sample of the same workload,
+    single-threaded and on all host cores."""
+    if name.startswith("sweep_"):
+        R, S = (int(x[1:]) for x in name.split("_")[1:])
+        w = wl.sweep(R, S, seed=seed)
+    else:
+        w = wl.by_name(name, seed=seed)
+    host = torch.empty((w.T, w.R, w.S), dtype=torch.int64, pin_memory=True)
+    w.fill(host.numpy().reshape(-1), threads=os.cpu_count() or 1)
+    d = host.to(device)
+    del host
+    st = sf.new_status(device)
+    e = lambda shape, dt: torch.empty(shape, dtype=dt, device=device)  # noqa: E731
+    fr = (e((w.T, w.S), torch.int64), e((w.T, w.S), torch.int32), e((w.T,), torch.int64))
+    frontier = lambda: sf.sf_frontier(d, a=fr[0], lead=fr[1], makespan=fr[2], status=st)  # noqa: E731
+    pipe = Pipeline(sf, w, d)
+    din = w.T * w.R * w.S * 8
+    rec = {"config": name, "R": w.R, "S": w.S, "T": w.T, "W": w.W, "gbytes": round(din / 1e9, 3)}
+    f_secs = timed_loop(frontier, steps, warmup, 1, device, True) / steps
+    f_bytes = din + w.T * w.S * 12 + w.T * 8
+    rec["frontier"] = {"ms": round(f_secs * 1e3, 4), "gbs": round(f_bytes / f_secs / 1e9, 1),
+                       "frac": round(f_bytes / f_secs / 1e9 / peak, 4), "records_per_s": w.records / f_secs}
+    a_secs = timed_loop(pipe.aggregate, steps, warmup, 1, device, True) / steps
+    a_bytes = pipe.algorithmic_bytes()["window_aggregate"]
+    rec["aggregate"] = {"ms": round(a_secs * 1e3, 4), "gbs": round(a_bytes / a_secs / 1e9, 1),
+                        "frac": round(a_bytes / a_secs / 1e9 / peak, 4)}
+    s_secs = timed_loop(pipe.step, steps, warmup, 1, device, True) / steps
+    rec["step"] = {"ms": round(s_secs * 1e3, 4), "records_per_s": w.records / s_secs}
+    torch.cuda.synchronize()
+    rec["status"] = int(st.item()) | int(pipe.status.item())
+    del d, pipe, fr
+    torch.cuda.empty_cache()
+    if oracle is not None:
+        n = max(1, ORACLE_SAMPLE_RECORDS // (w.R * w.S))
+        cores = os.cpu_count() or 1
+        one = oracle_rate(oracle, w, n, 1)
+        allc = oracle_rate(oracle, w, n, max(1, min(cores, w.T // n)))
+        rec["oracle"] = {"records_per_s_1core": one["value"], "records_per_s_all_cores": allc["value"],
+                         "cores": allc["cores"], "sample": allc["sample"] + " (single-core: the first slice)"}
+        rec["gpu_over_oracle_all_cores"] = round(rec["step"]["records_per_s"] / allc["value"], 1)
+    return rec
 
 
 def run_configs(args):
@@ -526,44 +682,10 @@ def run_configs(args):
     from paper_2606_06751_gb300 import stagefrontier as sf
 
     peak, peak_kind = peaks()
-    names = ["tiny", "ddp128", "fsdp1024", "accum8192"] + [f"sweep_R{R}_S{S}" for R in wl.SWEEP_R
-                                                           for S in wl.SWEEP_S]
+    names = CONFIG_NAMES
     if args.only:
         names = [n for n in names if n in args.only.split(",")]
-    out = []
-    for name in names:
-        if name.startswith("sweep_"):
-            R, S = (int(x[1:]) for x in name.split("_")[1:])
-            w = wl.sweep(R, S, seed=args.seed)
-        else:
-            w = wl.by_name(name, seed=args.seed)
-        host = torch.empty((w.T, w.R, w.S), dtype=torch.int64, pin_memory=True)
-        w.fill(host.numpy().reshape(-1), threads=os.cpu_count() or 1)
-        d = host.to(device)
-        del host
-        st = sf.new_status(device)
-        nW = sf.num_windows(0, w.T, w.W)
-        e = lambda shape, dt: torch.empty(shape, dtype=dt, device=device)  # noqa: E731
-        fr = (e((w.T, w.S), torch.int64), e((w.T, w.S), torch.int32), e((w.T,), torch.int64))
-        frontier = lambda: sf.sf_frontier(d, a=fr[0], lead=fr[1], makespan=fr[2], status=st)  # noqa: E731
-        pipe = Pipeline(sf, w, d)
-        din = w.T * w.R * w.S * 8
-        rec = {"config": name, "R": w.R, "S": w.S, "T": w.T, "W": w.W, "gbytes": round(din / 1e9, 3)}
-        f_secs = timed_loop(frontier, args.steps, args.warmup, 1, device, True) / args.steps
-        f_bytes = din + w.T * w.S * 12 + w.T * 8
-        rec["frontier"] = {"ms": round(f_secs * 1e3, 4), "gbs": round(f_bytes / f_secs / 1e9, 1),
-                           "frac": round(f_bytes / f_secs / 1e9 / peak, 4), "records_per_s": w.records / f_secs}
-        a_secs = timed_loop(pipe.aggregate, args.steps, args.warmup, 1, device, True) / args.steps
-        a_bytes = pipe.algorithmic_bytes()["window_aggregate"]
-        rec["aggregate"] = {"ms": round(a_secs * 1e3, 4), "gbs": round(a_bytes / a_secs / 1e9, 1),
-                            "frac": round(a_bytes / a_secs / 1e9 / peak, 4)}
-        s_secs = timed_loop(pipe.step, args.steps, args.warmup, 1, device, True) / args.steps
-        rec["step"] = {"ms": round(s_secs * 1e3, 4), "records_per_s": w.records / s_secs}
-        torch.cuda.synchronize()
-        rec["status"] = int(st.item()) | int(pipe.status.item())
-        out.append(rec)
-        del d, pipe, fr
-        torch.cuda.empty_cache()
+    out = [measure_config(n, sf, device, peak, args.steps, args.warmup, args.seed) for n in names]
     return {"metric": "per-configuration throughput (frontier pass, aggregation pass, whole step)",
             "unit": "GB/s and records/s", "peak_gbs": peak, "peak_kind": peak_kind, "steps": args.steps,
             "warmup": args.warmup, "configs": out}
@@ -579,8 +701,8 @@ def main(argv=None):
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--steps-override", type=int, default=None, help="shrink T (tests only)")
     ap.add_argument("--cpu-sample-windows", type=int, default=2)
-    ap.add_argument("--ref-sample-steps", type=int, default=100)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true", help="skip the per-configuration block")
     ap.add_argument("--configs", action="store_true",
                     help="throughput on every synthetic configuration instead of the benchmark step")
     ap.add_argument("--only", default=None, help="with --configs: comma-separated configuration names")

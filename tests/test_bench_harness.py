@@ -58,12 +58,14 @@ def test_timed_loop_takes_max_over_ranks():
 def test_reference_arm_line():
     out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
                           "--steps", "2", "--warmup", "3", "--workload", "ddp128", "--steps-override",
-                          "2000", "--ref-sample-steps", "200"],
+                          "2000"],
                          capture_output=True, text=True, timeout=600, cwd=ROOT)
     assert out.returncode == 0, out.stderr
     line = json.loads(out.stdout.strip().splitlines()[-1])
     assert line["impl"] == "reference" and line["unit"] == "records/s" and line["value"] > 0
-    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 1
+    # whole 1000-step windows, one per host thread: the two windows of 2000 steps
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == min(os.cpu_count(), 2)
+    assert line["config"]["W"] == 1000 and line["config"]["T"] == 2000
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
     assert line["higher_is_better"] is True and line["steps"] == 2
 
@@ -71,6 +73,6 @@ def test_reference_arm_line():
 def test_reference_arm_other_ranks_exit_quietly(monkeypatch):
     monkeypatch.setenv("RANK", "1")
     monkeypatch.setenv("WORLD_SIZE", "2")
-    args = bench.argparse.Namespace(workload="tiny", seed=0, steps_override=None, ref_sample_steps=10,
+    args = bench.argparse.Namespace(workload="tiny", seed=0, steps_override=None,
                                     warmup=3, steps=1)
     assert bench.run_reference(args) is None
