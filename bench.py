@@ -378,7 +378,7 @@ def run_ours(args):
         from oracle import oracle as O
         O.build_lib()
         configs = [measure_config(n, sf, device, peak, 5, 3, args.seed, oracle=O)
-                   for n in CONFIG_NAMES if n != w.name]
+                   for n in CONFIG_NAMES + FEW_STEP_NAMES if n != w.name]
 
     # end to end through the host-memory entry point: every step streams the
     # pinned host tensor to the GPU in 2000-step chunks (copies overlapping the
@@ -621,6 +621,9 @@ def run_reference(args):
 
 CONFIG_NAMES = ["tiny", "ddp128", "fsdp1024", "accum8192"] + [f"sweep_R{R}_S{S}" for R in wl.SWEEP_R
                                                                 for S in wl.SWEEP_S]
+# a single window of few steps over many ranks (the per-window use of Sec. 3):
+# fewer steps than SMs
+FEW_STEP_NAMES = ["steps_T100_R8192_S8", "steps_T8_R8192_S8", "steps_T1_R8192_S8", "steps_T64_R65536_S8"]
 ORACLE_SAMPLE_RECORDS = 4_000_000  # per oracle thread, per configuration
 
 
@@ -632,6 +635,9 @@ def measure_config(name: str, sf, device, peak: float, steps: int, warmup: int, 
     if name.startswith("sweep_"):
         R, S = (int(x[1:]) for x in name.split("_")[1:])
         w = wl.sweep(R, S, seed=seed)
+    elif name.startswith("steps_"):
+        T, R, S = (int(x[1:]) for x in name.split("_")[1:])
+        w = wl.sweep(R, S, seed=seed, steps=T)
     else:
         w = wl.by_name(name, seed=seed)
     host = torch.empty((w.T, w.R, w.S), dtype=torch.int64, pin_memory=True)
@@ -682,7 +688,7 @@ def run_configs(args):
     from paper_2606_06751_gb300 import stagefrontier as sf
 
     peak, peak_kind = peaks()
-    names = CONFIG_NAMES
+    names = CONFIG_NAMES + FEW_STEP_NAMES
     if args.only:
         names = [n for n in names if n in args.only.split(",")]
     out = [measure_config(n, sf, device, peak, args.steps, args.warmup, args.seed) for n in names]

@@ -146,10 +146,12 @@ sf_status sf_window_aggregate(const int64_t* d, int64_t T, int64_t R, int64_t S,
     return SF_EINVAL_ALIGN;
   const int64_t nW = sf_num_windows(t0, T, W);
   if (!accumulate) {
-    cudaError_t e = launch_zero(X, size_t(nW) * S * 8, stream);
-    if (e == cudaSuccess) e = launch_zero(D, size_t(nW) * 8, stream);
-    if (e == cudaSuccess && E) e = launch_zero(E, size_t(nW) * S * R * 8, stream);
-    if (e == cudaSuccess && C) e = launch_zero(C, size_t(nW) * S * R * 4, stream);
+    ZeroList z;
+    z.add(X, size_t(nW) * S * 8);
+    z.add(D, size_t(nW) * 8);
+    z.add(E, size_t(nW) * S * R * 8);
+    z.add(C, size_t(nW) * S * R * 4);
+    cudaError_t e = launch_zero_many(z, stream);
     if (e != cudaSuccess) return SF_ECUDA;
   }
   StreamJob j;
@@ -179,10 +181,12 @@ sf_status sf_window_baselines(const int64_t* d, int64_t T, int64_t R, int64_t S,
     return SF_EINVAL_ALIGN;
   const int64_t nW = sf_num_windows(t0, T, W);
   if (!accumulate) {
-    cudaError_t e = launch_zero(M, size_t(nW) * S * 8, stream);
-    if (e == cudaSuccess) e = launch_zero(SUM, size_t(nW) * S * 16, stream);
-    if (e == cudaSuccess) e = launch_zero(SLOW, size_t(nW) * S * 8, stream);
-    if (e == cudaSuccess) e = launch_zero(RANK0, size_t(nW) * S * 8, stream);
+    ZeroList z;
+    z.add(M, size_t(nW) * S * 8);
+    z.add(SUM, size_t(nW) * S * 16);
+    z.add(SLOW, size_t(nW) * S * 8);
+    z.add(RANK0, size_t(nW) * S * 8);
+    cudaError_t e = launch_zero_many(z, stream);
     if (e != cudaSuccess) return SF_ECUDA;
   }
   StreamJob j;
@@ -238,8 +242,10 @@ sf_status sf_rank_lag_windows(const int64_t* d, int64_t T, int64_t R, int64_t S,
     return SF_EINVAL_ALIGN;
   if (!workspace || !rank_workspace_ok(T, R, S, workspace_bytes)) return SF_EWORKSPACE;
   const size_t bytes = size_t(sf_num_windows(t0, T, W)) * S * 8;
-  if (!accumulate && ((Lw && launch_zero(Lw, bytes, stream) != cudaSuccess) ||
-                      (Gw && launch_zero(Gw, bytes, stream) != cudaSuccess)))
+  ZeroList z;
+  z.add(Lw, bytes);
+  z.add(Gw, bytes);
+  if (!accumulate && launch_zero_many(z, stream) != cudaSuccess)
     return SF_ECUDA;
   return cuda_status(launch_rank_select(d, T, R, S, 1, t0, W, nullptr, nullptr, nullptr, Lw, Gw, nullptr, workspace,
                                         workspace_bytes, status, stream));
@@ -258,8 +264,10 @@ sf_status sf_group_aggregate(const int64_t* d, int64_t T, int64_t R, int64_t S, 
   if (!aligned(d, 16) || !aligned(group, 4) || !aligned(Xg, 8) || !aligned(Dg, 8) || !aligned(status, 4))
     return SF_EINVAL_ALIGN;
   const size_t nW = size_t(sf_num_windows(t0, T, W));
-  if (!accumulate && (launch_zero(Xg, nW * G * S * 8, stream) != cudaSuccess ||
-                      launch_zero(Dg, nW * G * 8, stream) != cudaSuccess))
+  ZeroList z;
+  z.add(Xg, nW * G * S * 8);
+  z.add(Dg, nW * G * 8);
+  if (!accumulate && launch_zero_many(z, stream) != cudaSuccess)
     return SF_ECUDA;
   return cuda_status(launch_group_windows(d, T, R, S, group, G, t0, W, Xg, Dg, status, stream));
 }
@@ -320,12 +328,14 @@ sf_status sf_direct_gain(const int64_t* d, int64_t T, int64_t R, int64_t S, int6
       !aligned(D, 8) || !aligned(E, 8) || !aligned(C, 4) || !aligned(quality, 8) || !aligned(status, 4))
     return SF_EINVAL_ALIGN;
   const int64_t nW = (T + W - 1) / W;
-  cudaError_t e = launch_zero(X, size_t(nW) * S * 8, stream);
-  if (e == cudaSuccess) e = launch_zero(Y, size_t(nW) * S * 8, stream);
-  if (e == cudaSuccess) e = launch_zero(D, size_t(nW) * 8, stream);
-  if (e == cudaSuccess && E) e = launch_zero(E, size_t(nW) * S * R * 8, stream);
-  if (e == cudaSuccess && C) e = launch_zero(C, size_t(nW) * S * R * 4, stream);
-  if (e == cudaSuccess && quality) e = launch_zero(quality, size_t(nW) * 6 * 8, stream);
+  ZeroList z;
+  z.add(X, size_t(nW) * S * 8);
+  z.add(Y, size_t(nW) * S * 8);
+  z.add(D, size_t(nW) * 8);
+  z.add(E, size_t(nW) * S * R * 8);
+  z.add(C, size_t(nW) * S * R * 4);
+  z.add(quality, size_t(nW) * 6 * 8);
+  cudaError_t e = launch_zero_many(z, stream);
   if (e != cudaSuccess) return SF_ECUDA;
   StreamJob j;
   j.d = d;

@@ -53,6 +53,21 @@ int sm_count();                     // SMs of the current device (cached)
 void count_launch(uint64_t n = 1);  // bump the library's launch counter
 
 cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t stream);
+// Up to kZeroMax buffers (whole 4-byte words) cleared by one launch; null or empty entries are skipped.
+constexpr int kZeroMax = 6;
+struct ZeroList {
+  void* ptr[kZeroMax];
+  size_t words[kZeroMax];
+  int n = 0;
+  void add(void* p, size_t bytes) {
+    if (p && bytes) {
+      ptr[n] = p;
+      words[n] = bytes / 4;
+      ++n;
+    }
+  }
+};
+cudaError_t launch_zero_many(const ZeroList& z, cudaStream_t stream);
 cudaError_t launch_wait_selftest(uint64_t limit_ns, uint32_t* status, cudaStream_t stream);
 cudaError_t launch_stream_pass(const StreamJob& job, cudaStream_t stream);
 cudaError_t launch_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W,

@@ -23,6 +23,16 @@ __global__ void zero_kernel(uint32_t* __restrict__ p, size_t words) {
     p[i] = 0u;
 }
 
+// Clears up to kZeroMax buffers in one launch (a call's accumulators).
+__global__ void zero_many_kernel(const ZeroList z) {
+  for (int b = 0; b < z.n; ++b) {
+    uint32_t* __restrict__ p = static_cast<uint32_t*>(z.ptr[b]);
+    for (size_t i = blockIdx.x * size_t(blockDim.x) + threadIdx.x; i < z.words[b];
+         i += size_t(gridDim.x) * blockDim.x)
+      p[i] = 0u;
+  }
+}
+
 // ---------------------------------------------------------------------------
 // Lower median, one warp per column.  A CTA of 8 warps owns (window w, eight
 // consecutive flat columns c = r*S + s).  The window's rows of those columns
@@ -742,6 +752,16 @@ cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t stream) {
   const int grid = static_cast<int>(std::min<size_t>((words + 255) / 256, size_t(sm_count()) * 8));
   count_launch();
   zero_kernel<<<grid, 256, 0, stream>>>(static_cast<uint32_t*>(p), words);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_zero_many(const ZeroList& z, cudaStream_t stream) {
+  size_t words = 0;
+  for (int b = 0; b < z.n; ++b) words = std::max(words, z.words[b]);
+  if (words == 0) return cudaSuccess;
+  const int grid = static_cast<int>(std::min<size_t>((words + 255) / 256, size_t(sm_count()) * 8));
+  count_launch();
+  zero_many_kernel<<<grid, 256, 0, stream>>>(z);
   return cudaGetLastError();
 }
 

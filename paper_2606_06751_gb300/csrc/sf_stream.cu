@@ -27,6 +27,8 @@
 #include <numeric>
 #include <type_traits>
 
+#include <cooperative_groups.h>
+
 #include "sf_device.cuh"
 #include "sf_launch.h"
 
@@ -899,6 +901,110 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
 }
 
 // --------------------------------------------------------------------------
+// Few steps over many ranks (fewer steps than SMs: one window of a few
+// hundred steps, the per-window use of Sec. 3): each step's ranks are split
+// over a thread-block cluster of `csize` CTAs, so every SM streams.  CTA j of
+// the cluster reads ranks [j R / csize, (j+1) R / csize) with 16-byte loads
+// (four rows in flight per thread), reduces its packed per-stage keys
+// (F << 16 | 65535 - r) to shared memory, and the cluster's first CTA takes
+// the maximum over the cluster's keys through distributed shared memory
+// (ranks are disjoint, so the largest key still carries the lowest attaining
+// rank) and runs the step's epilogue.  No global scratch.
+constexpr int kSplitThreads = 256;
+constexpr int kSplitMaxCluster = 16;  // above 8: a non-portable cluster size, allowed per kernel
+
+template <int S>
+__global__ void __launch_bounds__(kSplitThreads) split_frontier_kernel(const int64_t* __restrict__ d, const Params p) {
+  namespace cg = cooperative_groups;
+  cg::cluster_group cl = cg::this_cluster();
+  __shared__ uint64_t wkey[kSplitThreads / 32][S];
+  __shared__ uint64_t ckey[S];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int csize = static_cast<int>(cl.num_blocks());
+  const int j = static_cast<int>(cl.block_rank());
+  const int64_t t = blockIdx.x / csize;
+  const int64_t R = p.R;
+  const int64_t r0 = R * j / csize, r1 = R * (j + 1) / csize;
+  const int64_t* dt = d + t * R * S;
+  FrontierRows<S> fr;
+  fr.init();
+  uint32_t dor = 0, tor = 0;
+  constexpr int U = 4;
+  for (int64_t r = r0 + threadIdx.x; r < r1; r += int64_t(kSplitThreads) * U) {
+    int64_t v[U][S];
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (r + int64_t(kSplitThreads) * u < r1) load_global_row<S>(dt + (r + int64_t(kSplitThreads) * u) * S, v[u]);
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (r + int64_t(kSplitThreads) * u < r1) fr.row(v[u], static_cast<int32_t>(r + kSplitThreads * u), dor, tor);
+  }
+#pragma unroll
+  for (int s = 0; s < S; ++s) {
+    const uint64_t km = warp_max_u64(fr.key(s));
+    if (lane == 0) wkey[warp][s] = km;
+  }
+  __syncthreads();
+  if (threadIdx.x < S) {
+    uint64_t k = 0;
+    for (int w = 0; w < kSplitThreads / 32; ++w) k = wkey[w][threadIdx.x] > k ? wkey[w][threadIdx.x] : k;
+    ckey[threadIdx.x] = k;
+  }
+  cl.sync();  // every CTA's keys are visible to the cluster
+  if (j == 0 && warp == 0) {
+    uint64_t key = 0;
+    if (lane < S)
+      for (int q = 0; q < csize; ++q) {
+        const uint64_t k = *cl.map_shared_rank(&ckey[lane], static_cast<unsigned>(q));
+        key = k > key ? k : key;
+      }
+    WinAcc acc;
+    finalize_frontier(p, S, t, key, lane, acc);
+    if (p.X) flush_window(p, S, acc, lane);
+  }
+  cl.sync();  // the other CTAs' shared memory stays alive until the first CTA has read it
+  const uint32_t bits = range_bits(__reduce_or_sync(kFull, dor), __reduce_or_sync(kFull, tor));
+  if (lane == 0) report(p.status, bits);
+}
+
+template <int S>
+cudaError_t launch_split(const int64_t* d, const Params& p, int csize, cudaStream_t stream) {
+  static bool ready = false;  // attribute set once per process (same on every GB300)
+  if (!ready) {
+    const cudaError_t e = cudaFuncSetAttribute(split_frontier_kernel<S>,
+                                               cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+    ready = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(csize);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(static_cast<unsigned>(p.T * csize));
+  cfg.blockDim = dim3(kSplitThreads);
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, split_frontier_kernel<S>, d, p);
+}
+
+cudaError_t dispatch_split(int S, const int64_t* d, const Params& p, int csize, cudaStream_t stream) {
+  switch (S) {
+    case 2: return launch_split<2>(d, p, csize, stream);
+    case 4: return launch_split<4>(d, p, csize, stream);
+    case 6: return launch_split<6>(d, p, csize, stream);
+    case 8: return launch_split<8>(d, p, csize, stream);
+    case 10: return launch_split<10>(d, p, csize, stream);
+    case 12: return launch_split<12>(d, p, csize, stream);
+    case 14: return launch_split<14>(d, p, csize, stream);
+    case 16: return launch_split<16>(d, p, csize, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+// --------------------------------------------------------------------------
 // Generic path: any S <= 32, any R; one CTA of 256 threads per step range.
 constexpr int kGenThreads = 256;
 
@@ -1087,6 +1193,20 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
                     (reinterpret_cast<uintptr_t>(j.d) % 16 == 0) &&
                     (!j.gain || reinterpret_cast<uintptr_t>(j.m) % 16 == 0);
   const int sms = sm_count();
+  // fewer steps than SMs over many ranks (frontier and aggregation): split
+  // each step's ranks over a cluster so that every SM streams
+  if (!j.gain && !j.base && j.T < sms && j.R >= 1024 && (j.S % 2 == 0) && j.S <= 16 &&
+      reinterpret_cast<uintptr_t>(j.d) % 16 == 0) {
+    int csize = 1;
+    while (csize < kSplitMaxCluster && j.T * csize * 2 <= 2 * sms && j.R / (csize * 2) >= 512) csize *= 2;
+    count_launch();
+    cudaError_t e = dispatch_split(static_cast<int>(j.S), j.d, p, csize, stream);
+    if (e != cudaSuccess && csize > 8) {  // a 16-CTA cluster that cannot be placed: portable size
+      cudaGetLastError();
+      e = dispatch_split(static_cast<int>(j.S), j.d, p, 8, stream);
+    }
+    return e;
+  }
   if (fast) {
     p.step_rows = step_rows;
     if (step_rows <= kR0MaxRows) {

@@ -122,6 +122,31 @@ def test_window_aggregate_parity(sf, T, R, S, t0, W):
         assert np.array_equal(host(getattr(g, name)), getattr(o, name)), name
 
 
+# fewer steps than SMs over many ranks: each step's ranks are split over a
+# thread-block cluster (up to 16 CTAs) and combined through distributed
+# shared memory; ragged rank splits included (R = 9000)
+@pytest.mark.parametrize("T,R,S", [(1, 8192, 8), (8, 8192, 8), (64, 8192, 8), (1, 65536, 8), (8, 65536, 8),
+                                   (64, 65536, 8), (3, 9000, 16), (100, 8192, 4), (20, 2048, 2)])
+@pytest.mark.parametrize("kind", ["lognormal", "ties"])
+def test_few_steps_split_ranks(sf, T, R, S, kind):
+    d_np = make(T, R, S, T * 31 + R + S, kind)
+    d = dev(d_np)
+    st = sf.new_status("cuda")
+    f = sf.sf_frontier(d, status=st)
+    t0, W = 3, 7
+    win = sf.sf_window_aggregate(d, W, t0=t0, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    o = O.frontier(d_np)
+    assert np.array_equal(host(f.a), o.a)
+    assert np.array_equal(host(f.lead), o.lead)
+    assert np.array_equal(host(f.makespan), o.makespan)
+    ow = O.windows(d_np, W, t0=t0)
+    assert np.array_equal(host(win.X), ow.X) and np.array_equal(host(win.D), ow.D)
+    assert np.array_equal(host(win.E), ow.E) and np.array_equal(host(win.C), ow.C)
+    assert np.array_equal(host(win.step_lead), ow.step_lead)
+
+
 def test_window_aggregate_chunked_accumulate(sf):
     T, R, S, W, chunk = 90, 64, 8, 25, 35
     d_np = make(T, R, S, 5, "lognormal")
