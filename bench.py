@@ -46,7 +46,10 @@ from synth import workloads as wl  # noqa: E402
 
 METRIC = "rank·step·stage records/sec and achieved HBM GB/s (% of GB300 peak)"
 UNIT = "records/s"
-KERNEL_SOURCES = ("sf_stream.cu", "sf_select.cu", "sf_device.cuh")
+# the sources each roofline kernel is compiled from: a recorded DRAM traffic
+# figure is valid only while their hash is the one it was captured with
+KERNEL_SOURCES = {"window_median": ("sf_select.cu", "sf_device.cuh"),
+                  "direct_gain": ("sf_stream.cu", "sf_device.cuh")}
 
 
 # --------------------------------------------------------------------------- distributed harness
@@ -181,9 +184,9 @@ def peaks():
         return 6800.0, "fallback"
 
 
-def kernel_source_sha() -> str:
+def kernel_source_sha(kernel: str) -> str:
     h = hashlib.sha256()
-    for f in KERNEL_SOURCES:
+    for f in KERNEL_SOURCES.get(kernel, ("sf_stream.cu", "sf_select.cu", "sf_device.cuh")):
         with open(os.path.join(ROOT, "paper_2606_06751_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -192,7 +195,7 @@ def kernel_source_sha() -> str:
 def profiled_traffic(kernel: str, workload: str):
     """DRAM bytes per launch recorded from an ncu capture in profiles/, valid
     only while the kernel sources are unchanged (matching source sha)."""
-    sha = kernel_source_sha()
+    sha = kernel_source_sha(kernel)
     pdir = os.path.join(ROOT, "profiles")
     if not os.path.isdir(pdir):
         return None

@@ -1197,8 +1197,9 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
   // each step's ranks over a cluster so that every SM streams
   if (!j.gain && !j.base && j.T < sms && j.R >= 1024 && (j.S % 2 == 0) && j.S <= 16 &&
       reinterpret_cast<uintptr_t>(j.d) % 16 == 0) {
-    int csize = 1;
-    while (csize < kSplitMaxCluster && j.T * csize * 2 <= 2 * sms && j.R / (csize * 2) >= 512) csize *= 2;
+    // about two CTAs per SM in all, at least 512 ranks per CTA
+    int csize = static_cast<int>(std::min<int64_t>(kSplitMaxCluster, std::max<int64_t>(1, 2 * sms / j.T)));
+    while (csize > 1 && j.R / csize < 512) --csize;
     count_launch();
     cudaError_t e = dispatch_split(static_cast<int>(j.S), j.d, p, csize, stream);
     if (e != cudaSuccess && csize > 8) {  // a 16-CTA cluster that cannot be placed: portable size
