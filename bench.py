@@ -81,8 +81,20 @@ def max_over_ranks(x: float, ws: int, device) -> float:
     return float(t.item())
 
 
-def timed_loop(step, K: int, W: int, ws: int, device, use_cuda: bool) -> float:
-    """Run W untimed then K timed steps; returns the max-over-ranks seconds."""
+# Device-side delay queued before the first timed event when `ahead` is set:
+# about 10 ms at the GB300's 2 GHz SM clock, longer than the host needs to
+# enqueue 20 steps of a few launches each.
+AHEAD_CYCLES = 20_000_000
+L2_FLUSH_BYTES = 256 << 20  # a read of twice the 129 MB L2 evicts every input line
+
+
+def timed_loop(step, K: int, W: int, ws: int, device, use_cuda: bool, ahead: bool = False) -> float:
+    """Run W untimed then K timed steps; returns the max-over-ranks seconds.
+
+    ahead: queue the K steps behind a device-side delay, so that the events
+    bracket back-to-back device execution even when one step's kernels take
+    less time than the host needs to launch them (launches of ~10-30 us on
+    inputs of a few MB); the delay itself lies before the first event."""
     for _ in range(W):
         step()
     if use_cuda:
@@ -92,6 +104,8 @@ def timed_loop(step, K: int, W: int, ws: int, device, use_cuda: bool) -> float:
         stream = torch.cuda.current_stream()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         torch.cuda.synchronize()
+        if ahead:
+            torch.cuda._sleep(AHEAD_CYCLES)
         e0.record(stream)
         for _ in range(K):
             step()
@@ -105,6 +119,32 @@ def timed_loop(step, K: int, W: int, ws: int, device, use_cuda: bool) -> float:
         secs = time.perf_counter() - t0
     barrier(ws)
     return max_over_ranks(secs, ws, device)
+
+
+def timed_loop_flushed(step, K: int, W: int, device) -> float:
+    """K steps on an input smaller than L2, each preceded by a read of
+    L2_FLUSH_BYTES so that it reads its input from HBM (a read, not a write:
+    the evicting lines are clean, so no write-back of the flush runs under
+    the timed step); a pair of events brackets each step alone, and
+    everything is queued behind a device-side delay so that no host gap
+    falls inside a pair.  Returns the summed seconds of the K steps (one GPU)."""
+    scratch = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.int32, device=device)
+    for _ in range(W):
+        scratch.sum()
+        step()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    torch.cuda._sleep(AHEAD_CYCLES)
+    for i in range(K):
+        scratch.sum()
+        ev[i][0].record(stream)
+        step()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    secs = sum(a.elapsed_time(b) for a, b in ev) / 1e3
+    del scratch
+    return secs
 
 
 # --------------------------------------------------------------------------- clocks
@@ -654,15 +694,22 @@ def measure_config(name: str, sf, device, peak: float, steps: int, warmup: int, 
     pipe = Pipeline(sf, w, d)
     din = w.T * w.R * w.S * 8
     rec = {"config": name, "R": w.R, "S": w.S, "T": w.T, "W": w.W, "gbytes": round(din / 1e9, 3)}
-    f_secs = timed_loop(frontier, steps, warmup, 1, device, True) / steps
+    if din < L2_FLUSH_BYTES:
+        # input smaller than twice the L2: every timed step after an L2 flush
+        rec["l2"] = f"input < 2 x L2: {L2_FLUSH_BYTES >> 20} MB read before each step, events around each step"
+        timed = lambda fn: timed_loop_flushed(fn, steps, warmup, device)  # noqa: E731
+    else:
+        rec["l2"] = "input > L2 on every pass; back-to-back steps queued ahead"
+        timed = lambda fn: timed_loop(fn, steps, warmup, 1, device, True, ahead=True)  # noqa: E731
+    f_secs = timed(frontier) / steps
     f_bytes = din + w.T * w.S * 12 + w.T * 8
     rec["frontier"] = {"ms": round(f_secs * 1e3, 4), "gbs": round(f_bytes / f_secs / 1e9, 1),
                        "frac": round(f_bytes / f_secs / 1e9 / peak, 4), "records_per_s": w.records / f_secs}
-    a_secs = timed_loop(pipe.aggregate, steps, warmup, 1, device, True) / steps
+    a_secs = timed(pipe.aggregate) / steps
     a_bytes = pipe.algorithmic_bytes()["window_aggregate"]
     rec["aggregate"] = {"ms": round(a_secs * 1e3, 4), "gbs": round(a_bytes / a_secs / 1e9, 1),
                         "frac": round(a_bytes / a_secs / 1e9 / peak, 4)}
-    s_secs = timed_loop(pipe.step, steps, warmup, 1, device, True) / steps
+    s_secs = timed(pipe.step) / steps
     rec["step"] = {"ms": round(s_secs * 1e3, 4), "records_per_s": w.records / s_secs}
     torch.cuda.synchronize()
     rec["status"] = int(st.item()) | int(pipe.status.item())

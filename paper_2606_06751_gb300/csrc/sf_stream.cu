@@ -24,6 +24,7 @@
 // Generic path (any other S <= 32 or R): one CTA per step range with plain
 // global loads.  Both paths share the per-step epilogues.
 #include <algorithm>
+#include <array>
 #include <numeric>
 #include <type_traits>
 
@@ -345,7 +346,7 @@ struct FrontierRows {
   }
 };
 
-constexpr int ceil_log2(int x) { return x <= 1 ? 0 : 1 + ceil_log2((x + 1) / 2); }
+__host__ __device__ constexpr int ceil_log2(int x) { return x <= 1 ? 0 : 1 + ceil_log2((x + 1) / 2); }
 
 // Evidence-pass maxima, with the frontier's lowest attaining rank.  A row
 // whose durations and medians are all below 2^kNarrowBits
@@ -901,6 +902,191 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
 }
 
 // --------------------------------------------------------------------------
+// Frontier pass over small steps (R*S <= 768, S in {2, 4, 8, 16}): G steps
+// share each warp instruction.  A warp splits into G groups of L = 32 / G
+// lanes; group g takes step kk0 + g of the warp's tile and lane j of the group
+// visits ranks j, j + L, ... in increasing order, so a strict '>' keeps the
+// lowest rank within a lane.  The per-stage packed keys (F << 16 | 65535 - r)
+// are then reduced over the group's L lanes by exchanges that halve the set of
+// keys a lane holds at each step (G steps' reductions in the instructions of
+// one), and the lanes j < S of each group run the step's epilogue for their
+// own step, so the per-step epilogue cost is shared by G steps as well.  The
+// tiles (K whole steps, K a multiple of G) arrive through the same warp-owned
+// ring stages as the other small-step path, from the same producer.  With
+// consecutive ranks in consecutive lanes, the 128-byte swizzle places the 16
+// or 8 lanes of a group on distinct 16-byte bank groups, so a group's row
+// reads are conflict free.
+template <int S, int L>
+__device__ __forceinline__ uint64_t group_max_keys(uint64_t (&k)[S], int j) {
+  static_assert(L >= S && (S & (S - 1)) == 0 && (L & (L - 1)) == 0, "L >= S, both powers of two");
+#pragma unroll
+  for (int lvl = 0; (L >> (lvl + 1)) >= 1; ++lvl) {
+    const int o = L >> (lvl + 1);
+    const int n = S >> lvl;  // keys this lane still holds
+    if (n > 1) {
+      // the lane with bit o set keeps the upper half of its keys, its partner the lower
+      const bool up = (j & o) != 0;
+#pragma unroll
+      for (int i = 0; i < n / 2; ++i) {
+        const uint64_t send = up ? k[i] : k[i + n / 2];
+        const uint64_t keep = up ? k[i + n / 2] : k[i];
+        const uint64_t got = __shfl_xor_sync(kFull, send, o);
+        k[i] = keep > got ? keep : got;
+      }
+    } else {
+      const uint64_t got = __shfl_xor_sync(kFull, k[0], o);
+      k[0] = k[0] > got ? k[0] : got;
+    }
+  }
+  // lane j now holds the group maximum of stage j >> (log2 L - log2 S)
+  return k[0];
+}
+
+// Frontier epilogue of one group's step t (the group's lanes j < S hold the
+// packed keys of stages j); the whole warp calls it, live = false for groups
+// past the tile's last step.
+template <int S, int L>
+__device__ __forceinline__ void finalize_group(const Params& p, int64_t t, uint64_t key, int j, bool live,
+                                               WinAcc& acc) {
+  const bool valid = live && j < S;
+  const int64_t F = valid ? static_cast<int64_t>(key >> 16) : 0;
+  const int32_t ld = valid ? 65535 - static_cast<int32_t>(key & 0xffffu) : 0;
+  int64_t Fprev = __shfl_up_sync(kFull, F, 1, L);
+  if (j == 0) Fprev = 0;  // F[t,-1] = 0
+  const int64_t a = valid ? F - Fprev : 0;
+  const int64_t mk = __shfl_sync(kFull, F, S - 1, L);
+  uint64_t km = 0;
+  if (p.X && p.step_lead) {
+    // leading stage: largest increment, lowest stage on ties
+    km = valid ? ((static_cast<uint64_t>(a) << 5) | static_cast<uint64_t>(31 - j)) : 0;
+#pragma unroll
+    for (int o = 1; o < S; o <<= 1) {
+      const uint64_t got = __shfl_xor_sync(kFull, km, o);
+      km = km > got ? km : got;
+    }
+  }
+  if (!live) return;
+  if (valid) {
+    if (p.a) p.a[t * S + j] = a;
+    if (p.lead) p.lead[t * S + j] = ld;
+  }
+  if (j == 0 && p.mk) p.mk[t] = mk;
+  if (p.X) {
+    const int64_t w = acc.wt.at(t, p.t0, p.W, p.w_first);
+    if (w != acc.cur) {
+      flush_window(p, S, acc, j);
+      acc.cur = w;
+    }
+    acc.x += a;
+    acc.dsum += mk;
+    if (valid && ld >= 0 && ld < p.R) {  // always true for valid input; guards flagged input
+      const int64_t idx = (w * S + j) * p.R + ld;
+      if (p.E && a != 0)
+        atomicAdd(reinterpret_cast<unsigned long long*>(&p.E[idx]), static_cast<unsigned long long>(a));
+      if (p.C) atomicAdd(&p.C[idx], 1);
+    }
+    if (p.step_lead && j == 0) p.step_lead[t] = static_cast<uint8_t>(31 - static_cast<int>(km & 31u));
+  }
+}
+
+template <int S, int G>
+__global__ void __launch_bounds__(kBlockThreads, 1)
+    lanes_kernel(const __grid_constant__ CUtensorMap map, const Params p) {
+  constexpr int L = 32 / G;
+  constexpr int U = S <= 8 ? 4 : 2;  // rank rows in flight per lane
+  constexpr int kShift = ceil_log2(L) - ceil_log2(S);
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* ring = align_1024(smem_raw);
+  uint64_t* full = reinterpret_cast<uint64_t*>(ring + kRingBytes);
+  uint64_t* empty = full + kMaxStages;
+  volatile int* abort = reinterpret_cast<volatile int*>(empty + kMaxStages);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t NB = gridDim.x, b = blockIdx.x;
+  const int64_t t_begin = p.T * b / NB, t_end = p.T * (b + 1) / NB;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kMaxStages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    *abort = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+
+  if (warp == kConsumerWarps) {
+    if (lane == 0) produce(&map, &map, p, t_begin, t_end, ring, full, empty, abort);
+    return;
+  }
+
+  const int g = lane / L, j = lane % L;
+  uint32_t dor = 0, tor = 0;
+  WinAcc acc;
+  const int R = static_cast<int>(p.R);
+  const int64_t n_local = t_end - t_begin;
+  const int64_t n_tiles = (n_local + p.K - 1) / p.K;
+  // one round: group g takes step kk of `tile` (step t of the pass)
+  auto round = [&](const unsigned char* tile, int kk, int64_t t, bool live, bool have) {
+    FrontierRows<S> rs;
+    rs.init();
+    if (have && live) {
+      const int q0 = kk * R;
+      for (int r0 = j; r0 < R; r0 += L * U) {
+        int64_t v[U][S];
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+          if (r0 + L * u < R) load_row<S, true>(tile, q0 + r0 + L * u, v[u]);
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+          if (r0 + L * u < R) rs.row(v[u], r0 + L * u, dor, tor);
+      }
+    }
+    uint64_t k[S];
+#pragma unroll
+    for (int s = 0; s < S; ++s) k[s] = rs.key(s);
+    const uint64_t ks = group_max_keys<S, L>(k, j);
+    // lane j < S of the group takes stage j's key from the lane holding it
+    const uint64_t mykey = __shfl_sync(kFull, ks, (j & (S - 1)) << kShift, L);
+    finalize_group<S, L>(p, t, mykey, j, live, acc);
+  };
+  // K steps per tile (a multiple of G): the warp's tiles one at a time, G steps per round
+  uint32_t i = 0;
+  for (int64_t jt = warp; jt < n_tiles; jt += kConsumerWarps, ++i) {
+    const uint32_t st = 2u * warp + (i & 1u), ph = (i >> 1) & 1u;
+    const bool have = mbar_wait_bounded(&full[st], ph, abort);
+    const unsigned char* tile = ring + size_t(st) * p.stage_bytes;
+    const int nsteps = static_cast<int>(min(int64_t(p.K), n_local - jt * p.K));
+    for (int kk0 = 0; kk0 < nsteps; kk0 += G) {
+      const int kk = kk0 + g;
+      round(tile, kk, t_begin + jt * p.K + kk, kk < nsteps, have);
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty[st]);
+  }
+
+  if (p.X) flush_window(p, S, acc, j);
+  const uint32_t bits = range_bits(__reduce_or_sync(kFull, dor), __reduce_or_sync(kFull, tor)) |
+                        (*abort ? SF_ST_TIMEOUT : 0u);
+  if (lane == 0) report(p.status, bits);
+}
+
+// Steps per warp instruction of the small-step frontier pass: the largest
+// G in {2, 4, 8} with L = 32 / G >= S and G whole steps in one ring stage;
+// 0 when the shape takes the one-step-per-warp path.  (Steps of 6-12 KB,
+// one per stage, stay there: a warp taking both of its stages in one round
+// has no copy of its own in flight, and the in-order producer then holds
+// every warp up; measured at less than half the one-step-per-warp rate.)
+int lanes_groups(int64_t R, int64_t S) {
+  if (S != 2 && S != 4 && S != 8 && S != 16) return 0;
+  const int64_t step_rows = R * S / 16;
+  int G = 0;
+  for (int c = 2; c <= 8; c *= 2)
+    if (32 / c >= S && c * step_rows <= kR0MaxRows) G = c;
+  return G;
+}
+
+// --------------------------------------------------------------------------
 // Few steps over many ranks (fewer steps than SMs: one window of a few
 // hundred steps, the per-window use of Sec. 3): each step's ranks are split
 // over a thread-block cluster of `csize` CTAs, so every SM streams.  CTA j of
@@ -988,6 +1174,62 @@ cudaError_t launch_split(const int64_t* d, const Params& p, int csize, cudaStrea
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, split_frontier_kernel<S>, d, p);
+}
+
+// Cluster size for T steps over R ranks: the largest size (<= 16, at least
+// 512 ranks per CTA) at which all T clusters are resident at once.  A
+// cluster is placed within one GPC, so sizes that do not divide a GPC's CTA
+// slots evenly fit fewer clusters than the SM count suggests, and a second
+// wave of clusters costs more than the parallelism gained (100 steps x 8192
+// ranks: 1, 3, 6 and 12 CTAs per step ran at 20.6, 21.9, 25.0 and 28.3 us).
+// The resident counts come from the occupancy calculator, once per process.
+template <int S>
+int split_cluster_size(int64_t T, int64_t R) {
+  static const std::array<int, kSplitMaxCluster + 1> fit = [] {
+    std::array<int, kSplitMaxCluster + 1> f{};
+    if (cudaFuncSetAttribute(split_frontier_kernel<S>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+        cudaSuccess) {
+      cudaGetLastError();
+      return f;
+    }
+    for (int c = 1; c <= kSplitMaxCluster; ++c) {
+      cudaLaunchConfig_t cfg = {};
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = static_cast<unsigned>(c);
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.gridDim = dim3(static_cast<unsigned>(c));
+      cfg.blockDim = dim3(kSplitThreads);
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, split_frontier_kernel<S>, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        n = 0;
+      }
+      f[c] = n;
+    }
+    return f;
+  }();
+  int best = 1;
+  for (int c = 2; c <= kSplitMaxCluster; ++c)
+    if (R / c >= 512 && fit[c] >= T) best = c;
+  return best;
+}
+
+int split_cluster(int S, int64_t T, int64_t R) {
+  switch (S) {
+    case 2: return split_cluster_size<2>(T, R);
+    case 4: return split_cluster_size<4>(T, R);
+    case 6: return split_cluster_size<6>(T, R);
+    case 8: return split_cluster_size<8>(T, R);
+    case 10: return split_cluster_size<10>(T, R);
+    case 12: return split_cluster_size<12>(T, R);
+    case 14: return split_cluster_size<14>(T, R);
+    case 16: return split_cluster_size<16>(T, R);
+    default: return 1;
+  }
 }
 
 cudaError_t dispatch_split(int S, const int64_t* d, const Params& p, int csize, cudaStream_t stream) {
@@ -1140,6 +1382,28 @@ cudaError_t dispatch_fast(int S, const CUtensorMap& map, const CUtensorMap& map_
 #undef SF_CASE
 }
 
+cudaError_t dispatch_lanes(int S, int G, const CUtensorMap& map, const Params& p, int grid, cudaStream_t stream) {
+#define SF_LANES(SV, GV)                                                                          \
+  if (S == SV && G == GV) {                                                                       \
+    cudaError_t e = cudaFuncSetAttribute(lanes_kernel<SV, GV>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
+                                         static_cast<int>(kSmemBytes));                          \
+    if (e != cudaSuccess) return e;                                                               \
+    lanes_kernel<SV, GV><<<grid, kBlockThreads, kSmemBytes, stream>>>(map, p);                     \
+    return cudaGetLastError();                                                                    \
+  }
+  SF_LANES(2, 2)
+  SF_LANES(2, 4)
+  SF_LANES(2, 8)
+  SF_LANES(4, 2)
+  SF_LANES(4, 4)
+  SF_LANES(4, 8)
+  SF_LANES(8, 2)
+  SF_LANES(8, 4)
+  SF_LANES(16, 2)
+#undef SF_LANES
+  return cudaErrorInvalidValue;
+}
+
 }  // namespace
 
 EncodeFn encode_fn() {
@@ -1197,9 +1461,7 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
   // each step's ranks over a cluster so that every SM streams
   if (!j.gain && !j.base && j.T < sms && j.R >= 1024 && (j.S % 2 == 0) && j.S <= 16 &&
       reinterpret_cast<uintptr_t>(j.d) % 16 == 0) {
-    // about two CTAs per SM in all, at least 512 ranks per CTA
-    int csize = static_cast<int>(std::min<int64_t>(kSplitMaxCluster, std::max<int64_t>(1, 2 * sms / j.T)));
-    while (csize > 1 && j.R / csize < 512) --csize;
+    const int csize = split_cluster(static_cast<int>(j.S), j.T, j.R);
     count_launch();
     cudaError_t e = dispatch_split(static_cast<int>(j.S), j.d, p, csize, stream);
     if (e != cudaSuccess && csize > 8) {  // a 16-CTA cluster that cannot be placed: portable size
@@ -1210,9 +1472,12 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
   }
   if (fast) {
     p.step_rows = step_rows;
+    // frontier and aggregation over small steps: several steps per warp instruction
+    const int lanes = (!j.gain && !j.base) ? lanes_groups(j.R, j.S) : 0;
     if (step_rows <= kR0MaxRows) {
       p.regime = 0;
       p.K = static_cast<int>(kR0MaxRows / step_rows);
+      if (lanes > 0) p.K = lanes * static_cast<int>(kR0MaxRows / (lanes * step_rows));  // whole rounds of G steps
       p.box_rows = static_cast<int>(p.K * step_rows);
       p.tiles_per_step = 0;
     } else {
@@ -1231,7 +1496,8 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
       p.tiles_per_step = static_cast<int>((step_rows + br - 1) / br);
       p.K = 0;
     }
-    const bool swz = (j.S == 4 || j.S == 8 || j.S == 16);
+    // the small-step frontier pass reads every shape it takes (S = 2 too) 128B-swizzled
+    const bool swz = (j.S == 4 || j.S == 8 || j.S == 16) || lanes > 0;
     auto encode = [&](CUtensorMap* out, const int64_t* base, int64_t rows) {
       const cuuint64_t gdim[2] = {16, static_cast<cuuint64_t>(rows)};
       const cuuint64_t gstride[1] = {kRowBytes};
@@ -1262,6 +1528,7 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
     const int64_t units = p.regime == 0 ? (j.T + p.K - 1) / p.K : j.T;
     const int grid = static_cast<int>(std::min<int64_t>(sms, units));
     count_launch();
+    if (lanes > 0) return dispatch_lanes(static_cast<int>(j.S), lanes, map, p, grid, stream);
     if (j.base) return dispatch_fast<2>(static_cast<int>(j.S), map, map_m, p, grid, stream);
     return j.gain ? dispatch_fast<1>(static_cast<int>(j.S), map, map_m, p, grid, stream)
                   : dispatch_fast<0>(static_cast<int>(j.S), map, map_m, p, grid, stream);

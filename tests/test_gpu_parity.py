@@ -62,7 +62,16 @@ SHAPES = [
 GROUPED = [(9, 520, 12), (6, 1000, 14), (4, 512, 8), (3000, 512, 4), (700, 768, 6), (301, 2048, 2)]
 
 
-@pytest.mark.parametrize("T,R,S", SHAPES + GROUPED[4:])
+# small steps (R*S <= 768, S in {2, 4, 8, 16}) taken G = 2, 4 or 8 steps per
+# warp instruction: every (S, G) pair, rank counts that are not a multiple of
+# the lanes per step, step counts that are not a multiple of the tile; the
+# last four are 6-12 KB steps next to that path (one step per warp)
+LANES = [(257, 376, 2), (300, 104, 2), (999, 40, 2), (211, 184, 4), (405, 52, 4), (333, 44, 4),
+         (150, 94, 8), (97, 64, 8), (260, 46, 8), (70, 48, 16), (88, 33, 16),
+         (45, 90, 16), (33, 180, 8), (50, 300, 4), (40, 696, 2)]
+
+
+@pytest.mark.parametrize("T,R,S", SHAPES + GROUPED[4:] + LANES)
 @pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal"])
 def test_frontier_parity(sf, T, R, S, kind):
     d_np = make(T, R, S, T * 131 + R * 7 + S, kind)
@@ -79,7 +88,7 @@ def test_frontier_parity(sf, T, R, S, kind):
 # Long step ranges: every CTA streams many tiles, so every ring stage is reused
 # many times (both regimes, both passes).
 LONG = [(200000, 8, 6), (20000, 64, 4), (8000, 128, 8), (3000, 512, 4), (1500, 1024, 10),
-        (600, 4096, 8)]
+        (600, 4096, 8), (30000, 94, 8), (60000, 40, 2)]
 
 
 @pytest.mark.parametrize("T,R,S", LONG)
@@ -109,7 +118,7 @@ def test_long_ranges_reuse_ring(sf, T, R, S):
     assert np.array_equal(host(ev.Y)[:2], O.direct_gain(d_np[:2 * W], W, m2))
 
 
-@pytest.mark.parametrize("T,R,S", SHAPES[:4] + SHAPES[5:9] + SHAPES[14:18] + GROUPED)
+@pytest.mark.parametrize("T,R,S", SHAPES[:4] + SHAPES[5:9] + SHAPES[14:18] + GROUPED + LANES)
 @pytest.mark.parametrize("t0,W", [(0, 7), (13, 10), (0, 1000)])
 def test_window_aggregate_parity(sf, T, R, S, t0, W):
     d_np = make(T, R, S, T + R + S + t0, "ties" if R < 100 else "lognormal")
