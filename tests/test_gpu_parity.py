@@ -64,10 +64,11 @@ GROUPED = [(9, 520, 12), (6, 1000, 14), (4, 512, 8), (3000, 512, 4), (700, 768, 
 
 # small steps (R*S <= 768, S in {2, 4, 8, 16}) taken G = 2, 4 or 8 steps per
 # warp instruction: every (S, G) pair, rank counts that are not a multiple of
-# the lanes per step, step counts that are not a multiple of the tile; the
-# last four are 6-12 KB steps next to that path (one step per warp)
+# the lanes per step, step counts that are not a multiple of the tile; then
+# 6-12 KB steps just past that path (one step per warp, every S)
 LANES = [(257, 376, 2), (300, 104, 2), (999, 40, 2), (211, 184, 4), (405, 52, 4), (333, 44, 4),
          (150, 94, 8), (97, 64, 8), (260, 46, 8), (70, 48, 16), (88, 33, 16),
+         (61, 53, 16), (77, 100, 8), (99, 236, 4), (45, 440, 2),
          (45, 90, 16), (33, 180, 8), (50, 300, 4), (40, 696, 2)]
 
 
@@ -88,7 +89,7 @@ def test_frontier_parity(sf, T, R, S, kind):
 # Long step ranges: every CTA streams many tiles, so every ring stage is reused
 # many times (both regimes, both passes).
 LONG = [(200000, 8, 6), (20000, 64, 4), (8000, 128, 8), (3000, 512, 4), (1500, 1024, 10),
-        (600, 4096, 8), (30000, 94, 8), (60000, 40, 2)]
+        (600, 4096, 8), (30000, 94, 8), (60000, 40, 2), (20000, 53, 16)]
 
 
 @pytest.mark.parametrize("T,R,S", LONG)
