@@ -421,7 +421,7 @@ def run_ours(args):
         from oracle import oracle as O
         O.build_lib()
         configs = [measure_config(n, sf, device, peak, 5, 3, args.seed, oracle=O)
-                   for n in CONFIG_NAMES + FEW_STEP_NAMES if n != w.name]
+                   for n in CONFIG_NAMES + FEW_STEP_NAMES + GENERIC_NAMES if n != w.name]
 
     # end to end through the host-memory entry point: every step streams the
     # pinned host tensor to the GPU in 2000-step chunks (copies overlapping the
@@ -667,6 +667,9 @@ CONFIG_NAMES = ["tiny", "ddp128", "fsdp1024", "accum8192"] + [f"sweep_R{R}_S{S}"
 # a single window of few steps over many ranks (the per-window use of Sec. 3):
 # fewer steps than SMs
 FEW_STEP_NAMES = ["steps_T100_R8192_S8", "steps_T8_R8192_S8", "steps_T1_R8192_S8", "steps_T64_R65536_S8"]
+# 1 GiB shapes outside the tiled streaming path (odd S with R*S not a multiple
+# of 16; more than 16 stages): the generic kernels
+GENERIC_NAMES = ["sweep_R1000_S5", "sweep_R512_S24"]
 ORACLE_SAMPLE_RECORDS = 4_000_000  # per oracle thread, per configuration
 
 
@@ -738,7 +741,7 @@ def run_configs(args):
     from paper_2606_06751_gb300 import stagefrontier as sf
 
     peak, peak_kind = peaks()
-    names = CONFIG_NAMES + FEW_STEP_NAMES
+    names = CONFIG_NAMES + FEW_STEP_NAMES + GENERIC_NAMES
     if args.only:
         names = [n for n in names if n in args.only.split(",")]
     out = [measure_config(n, sf, device, peak, args.steps, args.warmup, args.seed) for n in names]

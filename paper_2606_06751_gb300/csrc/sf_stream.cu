@@ -1248,9 +1248,12 @@ cudaError_t dispatch_split(int S, const int64_t* d, const Params& p, int csize, 
 
 // --------------------------------------------------------------------------
 // Generic path: any S <= 32, any R; one CTA of 256 threads per step range.
+// The per-stage state is sized by the bound SMAX >= S (4, 8, 16 or 32) and
+// every stage loop is unrolled to SMAX with an `s < S` guard, so the state
+// stays in registers.
 constexpr int kGenThreads = 256;
 
-template <int MODE>
+template <int SMAX, int MODE, bool VEC>
 __global__ void __launch_bounds__(kGenThreads)
     stream_generic_kernel(const int64_t* __restrict__ d, const Params p) {
   constexpr bool GAIN = MODE == 1;
@@ -1269,46 +1272,91 @@ __global__ void __launch_bounds__(kGenThreads)
   for (int64_t t = t_begin; t < t_end; ++t) {
     const int64_t w = GAIN ? qt.at(t, 0, p.W, 0) : 0;
     if (GAIN && p.quality) qual_window(p, qa, w, lane);
-    int64_t b0[32], b1[32];
-    int32_t br[32];
+    int64_t b0[SMAX], b1[SMAX];
+    int32_t br[SMAX];
     uint64_t slow = 0;
-    for (int s = 0; s < S; ++s) {
+#pragma unroll
+    for (int s = 0; s < SMAX; ++s) {
       b0[s] = BASE ? 0 : -1;
       b1[s] = 0;
       br[s] = 0;
     }
-    for (int64_t r = threadIdx.x; r < R; r += kGenThreads) {
-      const int64_t* row = d + (t * R + r) * S;
-      int64_t P = 0, other = 0;
-      for (int s = 0; s < S; ++s) {
-        const int64_t v = row[s];
-        dor |= hi32(v);
-        P += v;
-        if (s == p.other_stage) other = v;
+    if constexpr (!VEC) {
+      // one rank row at a time per thread, in increasing rank order (a strict
+      // '>' keeps the lowest rank), each duration loaded where it is used
+      for (int64_t r = threadIdx.x; r < R; r += kGenThreads) {
+        const int64_t* row = d + (t * R + r) * S;
+        int64_t P = 0, other = 0;
+#pragma unroll
+        for (int s = 0; s < SMAX; ++s) {
+          if (s >= S) break;
+          const int64_t v = __ldg(row + s);
+          dor |= hi32(v);
+          P += v;
+          if (s == p.other_stage) other = v;
+          if (BASE) {
+            b0[s] = v > b0[s] ? v : b0[s];
+            b1[s] += v;
+          } else if (P > b0[s]) {
+            b0[s] = P;
+            br[s] = static_cast<int32_t>(r);
+          }
+        }
+        tor |= hi32(P);
         if (BASE) {
-          b0[s] = v > b0[s] ? v : b0[s];
-          b1[s] += v;
-        } else if (P > b0[s]) {
-          b0[s] = P;
-          br[s] = static_cast<int32_t>(r);
+          const uint64_t k = (static_cast<uint64_t>(P) << 16) | static_cast<uint64_t>(65535 - r);
+          slow = k > slow ? k : slow;
+        }
+        if (GAIN) {
+          const int64_t* mr = p.m + (w * R + r) * S;
+#pragma unroll
+          for (int s = 0; s < SMAX; ++s) {
+            if (s >= S) break;
+            int64_t cut = __ldg(row + s) - __ldg(mr + s);
+            cut = cut > 0 ? cut : 0;
+            b1[s] = (P - cut) > b1[s] ? (P - cut) : b1[s];
+          }
+          if (p.quality) qual_row(p, qa, t, r, P, other, dor);
         }
       }
-      tor |= hi32(P);
-      if (BASE) {
-        const uint64_t k = (static_cast<uint64_t>(P) << 16) | static_cast<uint64_t>(65535 - r);
-        slow = k > slow ? k : slow;
-      }
-      if (GAIN) {
-        const int64_t* mr = p.m + (w * R + r) * S;
-        for (int s = 0; s < S; ++s) {
-          int64_t cut = row[s] - mr[s];
-          cut = cut > 0 ? cut : 0;
-          b1[s] = (P - cut) > b1[s] ? (P - cut) : b1[s];
+    } else {
+      // even S (frontier and baseline passes): rows start 16-byte aligned and
+      // are loaded whole with 16-byte loads, one row in flight per thread
+      static_assert(!GAIN, "the evidence pass loads durations where it uses them");
+      for (int64_t r = threadIdx.x; r < R; r += kGenThreads) {
+        const int64_t* row = d + (t * R + r) * S;
+        int64_t v[SMAX];
+#pragma unroll
+        for (int s = 0; s < SMAX; s += 2) {
+          if (s >= S) break;
+          const longlong2 x = __ldg(reinterpret_cast<const longlong2*>(row + s));
+          v[s] = x.x;
+          v[s + 1] = x.y;
         }
-        if (p.quality) qual_row(p, qa, t, r, P, other, dor);
+        int64_t P = 0;
+#pragma unroll
+        for (int s = 0; s < SMAX; ++s) {
+          if (s >= S) break;
+          dor |= hi32(v[s]);
+          P += v[s];
+          if (BASE) {
+            b0[s] = v[s] > b0[s] ? v[s] : b0[s];
+            b1[s] += v[s];
+          } else if (P > b0[s]) {
+            b0[s] = P;
+            br[s] = static_cast<int32_t>(r);
+          }
+        }
+        tor |= hi32(P);
+        if (BASE) {
+          const uint64_t k = (static_cast<uint64_t>(P) << 16) | static_cast<uint64_t>(65535 - r);
+          slow = k > slow ? k : slow;
+        }
       }
     }
-    for (int s = 0; s < S; ++s) {
+#pragma unroll
+    for (int s = 0; s < SMAX; ++s) {
+      if (s >= S) break;
       uint64_t k0;
       if (BASE) k0 = static_cast<uint64_t>(b0[s]);
       else k0 = b0[s] < 0 ? 0ull : (static_cast<uint64_t>(b0[s]) << 16) | static_cast<uint64_t>(65535 - br[s]);
@@ -1535,10 +1583,20 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
   }
   const int grid = static_cast<int>(std::min<int64_t>(int64_t(sms) * 4, j.T));
   count_launch();
-  if (j.base) stream_generic_kernel<2><<<grid, kGenThreads, 0, stream>>>(j.d, p);
-  else if (j.gain) stream_generic_kernel<1><<<grid, kGenThreads, 0, stream>>>(j.d, p);
-  else stream_generic_kernel<0><<<grid, kGenThreads, 0, stream>>>(j.d, p);
-  return cudaGetLastError();
+  const bool vec = j.S % 2 == 0;  // whole-row 16-byte loads (frontier and baseline passes)
+  auto generic = [&](auto smax) {
+    constexpr int SM = decltype(smax)::value;
+    if (j.gain) stream_generic_kernel<SM, 1, false><<<grid, kGenThreads, 0, stream>>>(j.d, p);
+    else if (j.base && vec) stream_generic_kernel<SM, 2, true><<<grid, kGenThreads, 0, stream>>>(j.d, p);
+    else if (j.base) stream_generic_kernel<SM, 2, false><<<grid, kGenThreads, 0, stream>>>(j.d, p);
+    else if (vec) stream_generic_kernel<SM, 0, true><<<grid, kGenThreads, 0, stream>>>(j.d, p);
+    else stream_generic_kernel<SM, 0, false><<<grid, kGenThreads, 0, stream>>>(j.d, p);
+    return cudaGetLastError();
+  };
+  if (j.S <= 4) return generic(std::integral_constant<int, 4>{});
+  if (j.S <= 8) return generic(std::integral_constant<int, 8>{});
+  if (j.S <= 16) return generic(std::integral_constant<int, 16>{});
+  return generic(std::integral_constant<int, 32>{});
 }
 
 }  // namespace sf
