@@ -145,16 +145,18 @@ sf_status sf_window_aggregate(const int64_t* d, int64_t T, int64_t R, int64_t S,
       !aligned(status, 4))
     return SF_EINVAL_ALIGN;
   const int64_t nW = sf_num_windows(t0, T, W);
+  bool cleared = false;
   if (!accumulate) {
     ZeroList z;
     z.add(X, size_t(nW) * S * 8);
     z.add(D, size_t(nW) * 8);
     z.add(E, size_t(nW) * S * R * 8);
     z.add(C, size_t(nW) * S * R * 4);
-    cudaError_t e = launch_zero_many(z, stream);
+    cudaError_t e = launch_zero_many(z, stream, &cleared);
     if (e != cudaSuccess) return SF_ECUDA;
   }
   StreamJob j;
+  j.after_clear = cleared;
   j.d = d;
   j.T = T;
   j.R = R;
@@ -180,16 +182,18 @@ sf_status sf_window_baselines(const int64_t* d, int64_t T, int64_t R, int64_t S,
       !aligned(status, 4))
     return SF_EINVAL_ALIGN;
   const int64_t nW = sf_num_windows(t0, T, W);
+  bool cleared = false;
   if (!accumulate) {
     ZeroList z;
     z.add(M, size_t(nW) * S * 8);
     z.add(SUM, size_t(nW) * S * 16);
     z.add(SLOW, size_t(nW) * S * 8);
     z.add(RANK0, size_t(nW) * S * 8);
-    cudaError_t e = launch_zero_many(z, stream);
+    cudaError_t e = launch_zero_many(z, stream, &cleared);
     if (e != cudaSuccess) return SF_ECUDA;
   }
   StreamJob j;
+  j.after_clear = cleared;
   j.d = d;
   j.T = T;
   j.R = R;
@@ -335,9 +339,11 @@ sf_status sf_direct_gain(const int64_t* d, int64_t T, int64_t R, int64_t S, int6
   z.add(E, size_t(nW) * S * R * 8);
   z.add(C, size_t(nW) * S * R * 4);
   z.add(quality, size_t(nW) * 6 * 8);
-  cudaError_t e = launch_zero_many(z, stream);
+  bool cleared = false;
+  cudaError_t e = launch_zero_many(z, stream, &cleared);
   if (e != cudaSuccess) return SF_ECUDA;
   StreamJob j;
+  j.after_clear = cleared;
   j.d = d;
   j.T = T;
   j.R = R;

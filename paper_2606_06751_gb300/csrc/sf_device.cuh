@@ -169,6 +169,17 @@ __device__ __forceinline__ void hist_find(const uint32_t* hist, uint32_t rem, in
   bins_find(h, rem, lane, digit, below);
 }
 
+// Programmatic dependent launch.  A kernel launched with programmatic stream
+// serialization may start while the previous kernel on its stream still runs,
+// once every CTA of that kernel has called griddep_launch_dependents() (or
+// has exited); griddep_wait() returns when the previous kernel has completed
+// and its memory operations are visible, and at once for a kernel launched
+// without that attribute.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ void report(uint32_t* status, uint32_t bits) {
   if (status != nullptr && bits != 0u) atomicOr(status, bits);
 }

@@ -36,6 +36,11 @@ struct StreamJob {
   uint32_t* status = nullptr;
   // routing-baseline pass (sf_window_baselines)
   bool base = false;
+  // the previous launch on the stream is this call's clear of its outputs
+  // (launch_zero_many): the pass is launched as its programmatic dependent,
+  // streaming its first tiles while the clear runs, and writes nothing
+  // before that clear has completed
+  bool after_clear = false;
   int64_t* bM = nullptr;
   uint64_t* bSUM = nullptr;
   int64_t* bSLOW = nullptr;
@@ -67,7 +72,10 @@ struct ZeroList {
     }
   }
 };
-cudaError_t launch_zero_many(const ZeroList& z, cudaStream_t stream);
+// *launched (when given) tells whether a kernel was enqueued: nothing is when
+// every entry is empty.  The clear lets the next launch on the stream start
+// early (programmatic dependent launch, StreamJob::after_clear).
+cudaError_t launch_zero_many(const ZeroList& z, cudaStream_t stream, bool* launched = nullptr);
 cudaError_t launch_wait_selftest(uint64_t limit_ns, uint32_t* status, cudaStream_t stream);
 cudaError_t launch_stream_pass(const StreamJob& job, cudaStream_t stream);
 cudaError_t launch_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W,

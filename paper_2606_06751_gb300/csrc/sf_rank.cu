@@ -81,8 +81,6 @@ __device__ __forceinline__ int64_t key_value(int64_t ref, uint32_t key) {
 // Programmatic dependent launch: the encode of chunk c+1 runs while the
 // select of chunk c does; each kernel waits for its predecessor in the stream
 // only where it must (see launch_rank_select).
-__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 __device__ __forceinline__ void discard_l2_line(const void* p) {
   asm volatile("discard.global.L2 [%0], 128;" ::"l"(p) : "memory");
@@ -217,8 +215,8 @@ __global__ void __launch_bounds__(kEncThreads) rank_encode_kernel(const RankPara
   // let this chunk's select launch, then finish only once the previous
   // chunk's select (which read the other scratch buffer) has finished, so
   // that this kernel's completion implies every earlier kernel's
-  pdl_launch_dependents();
-  pdl_wait();
+  griddep_launch_dependents();
+  griddep_wait();
 }
 
 // Encode with a rank row split over SC/2 lanes (SC = 4, 8 or 16): lane j of a
@@ -378,8 +376,8 @@ __global__ void __launch_bounds__(kEncThreads) rank_encode_split_kernel(const Ra
   }
   const uint32_t bits = range_bits(__reduce_or_sync(kFull, dor), p.of_prefix ? __reduce_or_sync(kFull, tor) : 0u);
   if (lane == 0) report(p.status, bits);
-  pdl_launch_dependents();
-  pdl_wait();
+  griddep_launch_dependents();
+  griddep_wait();
 }
 
 // ------------------------------------------------------------------ select
@@ -528,8 +526,8 @@ __global__ void __launch_bounds__(kSelThreads, kSelPerSM) rank_select_kernel(con
   const int64_t tasks = p.Tc * S;
   // this chunk's encode (and, through its own wait, every earlier kernel) is
   // complete and visible; then the next chunk's encode may start
-  pdl_wait();
-  pdl_launch_dependents();
+  griddep_wait();
+  griddep_launch_dependents();
   for (int64_t task = blockIdx.x; task < tasks; task += gridDim.x) {
     const int64_t tl = task / S;
     const int s = static_cast<int>(task - tl * S);

@@ -23,8 +23,11 @@ __global__ void zero_kernel(uint32_t* __restrict__ p, size_t words) {
     p[i] = 0u;
 }
 
-// Clears up to kZeroMax buffers in one launch (a call's accumulators).
+// Clears up to kZeroMax buffers in one launch (a call's accumulators), and
+// lets the pass that follows it on the stream start at once (it waits for
+// this kernel's completion before its first write).
 __global__ void zero_many_kernel(const ZeroList z) {
+  griddep_launch_dependents();
   for (int b = 0; b < z.n; ++b) {
     uint32_t* __restrict__ p = static_cast<uint32_t*>(z.ptr[b]);
     for (size_t i = blockIdx.x * size_t(blockDim.x) + threadIdx.x; i < z.words[b];
@@ -755,10 +758,12 @@ cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_zero_many(const ZeroList& z, cudaStream_t stream) {
+cudaError_t launch_zero_many(const ZeroList& z, cudaStream_t stream, bool* launched) {
   size_t words = 0;
   for (int b = 0; b < z.n; ++b) words = std::max(words, z.words[b]);
+  if (launched) *launched = false;
   if (words == 0) return cudaSuccess;
+  if (launched) *launched = true;
   const int grid = static_cast<int>(std::min<size_t>((words + 255) / 256, size_t(sm_count()) * 8));
   count_launch();
   zero_many_kernel<<<grid, 256, 0, stream>>>(z);

@@ -622,6 +622,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
     if (lane == 0) produce(&map, &map_m, p, t_begin, t_end, ring, full, empty, abort);
     return;
   }
+  griddep_wait();  // outputs cleared by the launch before this one (when it is its dependent)
 
   uint32_t dor = 0, tor = 0;  // OR of duration / rank-total high words
   WinAcc acc;
@@ -1019,6 +1020,7 @@ __global__ void __launch_bounds__(kBlockThreads, 1)
     if (lane == 0) produce(&map, &map, p, t_begin, t_end, ring, full, empty, abort);
     return;
   }
+  griddep_wait();  // outputs cleared by the launch before this one (when it is its dependent)
 
   const int g = lane / L, j = lane % L;
   uint32_t dor = 0, tor = 0;
@@ -1138,6 +1140,7 @@ __global__ void __launch_bounds__(kSplitThreads) split_frontier_kernel(const int
   }
   cl.sync();  // every CTA's keys are visible to the cluster
   if (j == 0 && warp == 0) {
+    griddep_wait();  // outputs cleared by the launch before this one (when it is its dependent)
     uint64_t key = 0;
     if (lane < S)
       for (int q = 0; q < csize; ++q) {
@@ -1154,7 +1157,7 @@ __global__ void __launch_bounds__(kSplitThreads) split_frontier_kernel(const int
 }
 
 template <int S>
-cudaError_t launch_split(const int64_t* d, const Params& p, int csize, cudaStream_t stream) {
+cudaError_t launch_split(const int64_t* d, const Params& p, int csize, cudaStream_t stream, bool pdl) {
   static bool ready = false;  // attribute set once per process (same on every GB300)
   if (!ready) {
     const cudaError_t e = cudaFuncSetAttribute(split_frontier_kernel<S>,
@@ -1163,16 +1166,18 @@ cudaError_t launch_split(const int64_t* d, const Params& p, int csize, cudaStrea
     ready = true;
   }
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = static_cast<unsigned>(csize);
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see launch_ex
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.gridDim = dim3(static_cast<unsigned>(p.T * csize));
   cfg.blockDim = dim3(kSplitThreads);
   cfg.stream = stream;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = pdl ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, split_frontier_kernel<S>, d, p);
 }
 
@@ -1232,16 +1237,16 @@ int split_cluster(int S, int64_t T, int64_t R) {
   }
 }
 
-cudaError_t dispatch_split(int S, const int64_t* d, const Params& p, int csize, cudaStream_t stream) {
+cudaError_t dispatch_split(int S, const int64_t* d, const Params& p, int csize, cudaStream_t stream, bool pdl) {
   switch (S) {
-    case 2: return launch_split<2>(d, p, csize, stream);
-    case 4: return launch_split<4>(d, p, csize, stream);
-    case 6: return launch_split<6>(d, p, csize, stream);
-    case 8: return launch_split<8>(d, p, csize, stream);
-    case 10: return launch_split<10>(d, p, csize, stream);
-    case 12: return launch_split<12>(d, p, csize, stream);
-    case 14: return launch_split<14>(d, p, csize, stream);
-    case 16: return launch_split<16>(d, p, csize, stream);
+    case 2: return launch_split<2>(d, p, csize, stream, pdl);
+    case 4: return launch_split<4>(d, p, csize, stream, pdl);
+    case 6: return launch_split<6>(d, p, csize, stream, pdl);
+    case 8: return launch_split<8>(d, p, csize, stream, pdl);
+    case 10: return launch_split<10>(d, p, csize, stream, pdl);
+    case 12: return launch_split<12>(d, p, csize, stream, pdl);
+    case 14: return launch_split<14>(d, p, csize, stream, pdl);
+    case 16: return launch_split<16>(d, p, csize, stream, pdl);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -1269,6 +1274,7 @@ __global__ void __launch_bounds__(kGenThreads)
   QualAcc qa;
   WinTrack qt;  // window of the step a warp is on (evidence pass)
   BaseAcc bacc;
+  griddep_wait();  // outputs cleared by the launch before this one (when it is its dependent)
   for (int64_t t = t_begin; t < t_end; ++t) {
     const int64_t w = GAIN ? qt.at(t, 0, p.W, 0) : 0;
     if (GAIN && p.quality) qual_window(p, qa, w, lane);
@@ -1399,6 +1405,26 @@ __global__ void __launch_bounds__(kGenThreads)
 
 // --------------------------------------------------------------------------
 // Host side
+
+// Launch `kern` on `stream`; with `pdl`, as the programmatic dependent of the
+// previous launch on the stream (this call's clear of its outputs: the kernel
+// streams its first tiles while the clear runs and writes after griddep_wait).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_ex(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream, bool pdl,
+                      Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 template <int S, int MODE>
 cudaError_t prepare_fast() {
   return cudaFuncSetAttribute(stream_kernel<S, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1407,13 +1433,12 @@ cudaError_t prepare_fast() {
 
 template <int MODE>
 cudaError_t dispatch_fast(int S, const CUtensorMap& map, const CUtensorMap& map_m, const Params& p, int grid,
-                          cudaStream_t stream) {
-#define SF_CASE(SV)                                                                          \
-  case SV: {                                                                                 \
-    cudaError_t e = prepare_fast<SV, MODE>();                                     \
-    if (e != cudaSuccess) return e;                                                          \
-    stream_kernel<SV, MODE><<<grid, kBlockThreads, kSmemBytes, stream>>>(map, map_m, p);     \
-    return cudaGetLastError();                                                               \
+                          cudaStream_t stream, bool pdl) {
+#define SF_CASE(SV)                                                                                    \
+  case SV: {                                                                                           \
+    cudaError_t e = prepare_fast<SV, MODE>();                                                          \
+    if (e != cudaSuccess) return e;                                                                    \
+    return launch_ex(stream_kernel<SV, MODE>, grid, kBlockThreads, kSmemBytes, stream, pdl, map, map_m, p); \
   }
   switch (S) {
     SF_CASE(2)
@@ -1430,14 +1455,14 @@ cudaError_t dispatch_fast(int S, const CUtensorMap& map, const CUtensorMap& map_
 #undef SF_CASE
 }
 
-cudaError_t dispatch_lanes(int S, int G, const CUtensorMap& map, const Params& p, int grid, cudaStream_t stream) {
+cudaError_t dispatch_lanes(int S, int G, const CUtensorMap& map, const Params& p, int grid, cudaStream_t stream,
+                           bool pdl) {
 #define SF_LANES(SV, GV)                                                                          \
   if (S == SV && G == GV) {                                                                       \
     cudaError_t e = cudaFuncSetAttribute(lanes_kernel<SV, GV>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
                                          static_cast<int>(kSmemBytes));                          \
     if (e != cudaSuccess) return e;                                                               \
-    lanes_kernel<SV, GV><<<grid, kBlockThreads, kSmemBytes, stream>>>(map, p);                     \
-    return cudaGetLastError();                                                                    \
+    return launch_ex(lanes_kernel<SV, GV>, grid, kBlockThreads, kSmemBytes, stream, pdl, map, p);   \
   }
   SF_LANES(2, 2)
   SF_LANES(2, 4)
@@ -1511,10 +1536,10 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
       reinterpret_cast<uintptr_t>(j.d) % 16 == 0) {
     const int csize = split_cluster(static_cast<int>(j.S), j.T, j.R);
     count_launch();
-    cudaError_t e = dispatch_split(static_cast<int>(j.S), j.d, p, csize, stream);
+    cudaError_t e = dispatch_split(static_cast<int>(j.S), j.d, p, csize, stream, j.after_clear);
     if (e != cudaSuccess && csize > 8) {  // a 16-CTA cluster that cannot be placed: portable size
       cudaGetLastError();
-      e = dispatch_split(static_cast<int>(j.S), j.d, p, 8, stream);
+      e = dispatch_split(static_cast<int>(j.S), j.d, p, 8, stream, j.after_clear);
     }
     return e;
   }
@@ -1576,22 +1601,23 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
     const int64_t units = p.regime == 0 ? (j.T + p.K - 1) / p.K : j.T;
     const int grid = static_cast<int>(std::min<int64_t>(sms, units));
     count_launch();
-    if (lanes > 0) return dispatch_lanes(static_cast<int>(j.S), lanes, map, p, grid, stream);
-    if (j.base) return dispatch_fast<2>(static_cast<int>(j.S), map, map_m, p, grid, stream);
-    return j.gain ? dispatch_fast<1>(static_cast<int>(j.S), map, map_m, p, grid, stream)
-                  : dispatch_fast<0>(static_cast<int>(j.S), map, map_m, p, grid, stream);
+    const bool pdl = j.after_clear;
+    if (lanes > 0) return dispatch_lanes(static_cast<int>(j.S), lanes, map, p, grid, stream, pdl);
+    if (j.base) return dispatch_fast<2>(static_cast<int>(j.S), map, map_m, p, grid, stream, pdl);
+    return j.gain ? dispatch_fast<1>(static_cast<int>(j.S), map, map_m, p, grid, stream, pdl)
+                  : dispatch_fast<0>(static_cast<int>(j.S), map, map_m, p, grid, stream, pdl);
   }
   const int grid = static_cast<int>(std::min<int64_t>(int64_t(sms) * 4, j.T));
   count_launch();
   const bool vec = j.S % 2 == 0;  // whole-row 16-byte loads (frontier and baseline passes)
   auto generic = [&](auto smax) {
     constexpr int SM = decltype(smax)::value;
-    if (j.gain) stream_generic_kernel<SM, 1, false><<<grid, kGenThreads, 0, stream>>>(j.d, p);
-    else if (j.base && vec) stream_generic_kernel<SM, 2, true><<<grid, kGenThreads, 0, stream>>>(j.d, p);
-    else if (j.base) stream_generic_kernel<SM, 2, false><<<grid, kGenThreads, 0, stream>>>(j.d, p);
-    else if (vec) stream_generic_kernel<SM, 0, true><<<grid, kGenThreads, 0, stream>>>(j.d, p);
-    else stream_generic_kernel<SM, 0, false><<<grid, kGenThreads, 0, stream>>>(j.d, p);
-    return cudaGetLastError();
+    const bool pdl = j.after_clear;
+    if (j.gain) return launch_ex(stream_generic_kernel<SM, 1, false>, grid, kGenThreads, 0, stream, pdl, j.d, p);
+    if (j.base && vec) return launch_ex(stream_generic_kernel<SM, 2, true>, grid, kGenThreads, 0, stream, pdl, j.d, p);
+    if (j.base) return launch_ex(stream_generic_kernel<SM, 2, false>, grid, kGenThreads, 0, stream, pdl, j.d, p);
+    if (vec) return launch_ex(stream_generic_kernel<SM, 0, true>, grid, kGenThreads, 0, stream, pdl, j.d, p);
+    return launch_ex(stream_generic_kernel<SM, 0, false>, grid, kGenThreads, 0, stream, pdl, j.d, p);
   };
   if (j.S <= 4) return generic(std::integral_constant<int, 4>{});
   if (j.S <= 8) return generic(std::integral_constant<int, 8>{});
