@@ -102,12 +102,13 @@ __device__ __forceinline__ uint32_t hi32(int64_t v) {
 
 // --------------------------------------------------------------------------
 // Window index of step t, (t0 + t) / W - w_first, recomputed (one 64-bit
-// division) only when t leaves the last window seen: the steps a thread
-// visits increase, so that happens once per window rather than once per step.
+// division) only when t passes the end of the last window seen: every thread
+// visits its steps in increasing order, so that happens once per window
+// rather than once per step.
 struct WinTrack {
   int64_t lo = 0, hi = 0, w = 0;  // steps [lo, hi) belong to window w
   __device__ __forceinline__ int64_t at(int64_t t, int64_t t0, int64_t W, int64_t w_first) {
-    if (t < lo || t >= hi) {
+    if (t >= hi) {
       w = (t0 + t) / W - w_first;
       lo = (w + w_first) * W - t0;
       hi = lo + W;
@@ -121,6 +122,7 @@ struct WinTrack {
 struct WinAcc {
   int64_t cur = -1;
   int64_t x = 0, y = 0, dsum = 0;
+  int64_t erow = 0;  // E / C index of (window cur, this lane's stage, rank 0)
   WinTrack wt;
 };
 
@@ -161,11 +163,12 @@ __device__ __forceinline__ void finalize_frontier(const Params& p, int S, int64_
     if (w != acc.cur) {
       flush_window(p, S, acc, lane);
       acc.cur = w;
+      acc.erow = (w * S + lane) * p.R;
     }
     acc.x += a;
     acc.dsum += mk;
     if (valid && ld >= 0 && ld < p.R) {  // always true for valid input; guards flagged input
-      const int64_t idx = (w * S + lane) * p.R + ld;
+      const int64_t idx = acc.erow + ld;
       if (p.E && a != 0)
         atomicAdd(reinterpret_cast<unsigned long long*>(&p.E[idx]), static_cast<unsigned long long>(a));
       if (p.C) atomicAdd(&p.C[idx], 1);
@@ -204,12 +207,13 @@ __device__ __forceinline__ void finalize_gain(const Params& p, int S, int64_t t,
   if (w != acc.cur) {
     flush_window(p, S, acc, lane);
     acc.cur = w;
+    acc.erow = (w * S + lane) * p.R;
   }
   acc.x += a;
   acc.y += y;
   acc.dsum += FS;
   if (valid && ld >= 0 && ld < p.R) {  // lead-rank credit (always in range for valid input)
-    const int64_t idx = (w * S + lane) * p.R + ld;
+    const int64_t idx = acc.erow + ld;
     if (p.E && a != 0)
       atomicAdd(reinterpret_cast<unsigned long long*>(&p.E[idx]), static_cast<unsigned long long>(a));
     if (p.C) atomicAdd(&p.C[idx], 1);
@@ -977,11 +981,12 @@ __device__ __forceinline__ void finalize_group(const Params& p, int64_t t, uint6
     if (w != acc.cur) {
       flush_window(p, S, acc, j);
       acc.cur = w;
+      acc.erow = (w * S + j) * p.R;
     }
     acc.x += a;
     acc.dsum += mk;
     if (valid && ld >= 0 && ld < p.R) {  // always true for valid input; guards flagged input
-      const int64_t idx = (w * S + j) * p.R + ld;
+      const int64_t idx = acc.erow + ld;
       if (p.E && a != 0)
         atomicAdd(reinterpret_cast<unsigned long long*>(&p.E[idx]), static_cast<unsigned long long>(a));
       if (p.C) atomicAdd(&p.C[idx], 1);
