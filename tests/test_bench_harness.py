@@ -76,3 +76,20 @@ def test_reference_arm_other_ranks_exit_quietly(monkeypatch):
     args = bench.argparse.Namespace(workload="tiny", seed=0, steps_override=None,
                                     warmup=3, steps=1)
     assert bench.run_reference(args) is None
+
+
+def test_fractions_carry_the_nominal_rate_beside_the_measured_copy():
+    """Every record with GB/s and `frac` also gets `frac_nominal` (GB/s over the
+    nominal 8000 GB/s), in nested records and lists; other fields are left alone."""
+    line = {"roofline": {"achieved": 5780.0, "frac": 0.8537},
+            "lag_pass": {"gbs": 2816.0, "frac": 0.416},
+            "configs": [{"frontier": {"gbs": 6400.0, "frac": 0.945}, "aggregate": {"gbs": 4000.0, "frac": 0.59}}],
+            "e2e": {"h2d_gbs": 150.0, "frac_of_link": 1.0}}
+    out = bench.add_nominal(line, 6770.5, "measured")
+    assert out["roofline"]["frac_nominal"] == round(5780.0 / 8000.0, 4)
+    assert out["lag_pass"]["frac_nominal"] == round(2816.0 / 8000.0, 4)
+    assert out["configs"][0]["frontier"]["frac_nominal"] == 0.8
+    assert out["configs"][0]["aggregate"]["frac_nominal"] == 0.5
+    assert "frac_nominal" not in out["e2e"]
+    rec = bench.peaks_record(6770.5, "measured")
+    assert "6770.5" in rec["frac"] and "8000" in rec["frac_nominal"]
