@@ -300,6 +300,8 @@ class Pipeline:
                                  e((nW, S), torch.int64))
         self.lag = sf.Lag(e((T, S), torch.int64), e((T, S), torch.int64), e((T, S), torch.int64))
         self.spread = e((nW, S), torch.int64)
+        self.fr_a = e((T, S), torch.int64)    # frontier increments, input of the tie-set pass
+        self.ties = e((T, S), torch.int32)
         self.rank_ws = sf.rank_workspace(T, R, S, dev)
         # role groups: nodes of 128 consecutive ranks (one group when R <= 128)
         self.n_groups = max(1, R // 128)
@@ -347,6 +349,11 @@ class Pipeline:
         """The raw rank spread per window (sf_raw_spread)."""
         self.sf.sf_raw_spread(self.d, self.w.W, spread=self.spread, workspace=self.rank_ws, status=self.status)
 
+    def frontier_ties(self):
+        """Size of the lead rank's tie set per step and stage (sf_frontier_ties),
+        on the increments of an earlier sf_frontier call."""
+        self.sf.sf_frontier_ties(self.d, a=self.fr_a, ties=self.ties, status=self.status)
+
     def group_aggregate(self):
         """The frontier within node groups of 128 ranks (sf_group_aggregate)."""
         self.sf.sf_group_aggregate(self.d, self.node_group, self.n_groups, self.w.W, out=self.grp,
@@ -369,6 +376,7 @@ class Pipeline:
             "rank_lag": din + 3 * w.T * w.S * 8,
             "raw_spread": din + nW * w.S * 8,
             "group_aggregate": din + w.R * 4 + nW * self.n_groups * (w.S + 1) * 8,
+            "frontier_ties": din + w.T * w.S * (8 + 4),
         }
 
 
@@ -420,6 +428,8 @@ def run_ours(args):
     lag_secs = timed_loop(pipe.rank_lag, args.steps, args.warmup, ws, device, True) / args.steps
     spread_secs = timed_loop(pipe.raw_spread, args.steps, args.warmup, ws, device, True) / args.steps
     group_secs = timed_loop(pipe.group_aggregate, args.steps, args.warmup, ws, device, True) / args.steps
+    sf.sf_frontier(d, a=pipe.fr_a, status=pipe.status, outputs=("a",))
+    ties_secs = timed_loop(pipe.frontier_ties, args.steps, args.warmup, ws, device, True) / args.steps
 
     # rank-major ingest: the same steps as the gather delivers them (one
     # [R][n][S] block per window), converted back into d in place of itself
@@ -544,6 +554,9 @@ def run_ours(args):
         "group_pass": {"entry": "sf_group_aggregate", "groups": pipe.n_groups, "ms": round(group_secs * 1e3, 4),
                        "gbs": round(algo["group_aggregate"] / group_secs / 1e9, 1),
                        "frac": round(algo["group_aggregate"] / group_secs / 1e9 / peak, 4)},
+        "ties_pass": {"entry": "sf_frontier_ties", "ms": round(ties_secs * 1e3, 4),
+                      "gbs": round(algo["frontier_ties"] / ties_secs / 1e9, 1),
+                      "frac": round(algo["frontier_ties"] / ties_secs / 1e9 / peak, 4)},
         "ingest_pass": {"entry": "sf_gathered_to_steps", "ms": round(ingest_secs * 1e3, 4),
                         "gbs": round(2 * w.nbytes / ingest_secs / 1e9, 1),
                         "frac": round(2 * w.nbytes / ingest_secs / 1e9 / peak, 4)},

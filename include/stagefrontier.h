@@ -102,6 +102,24 @@ sf_status sf_frontier(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t
                       int64_t* makespan, uint32_t* status, cudaStream_t stream);
 
 /*
+ * sf_frontier_ties - the size of the lead rank's tie set, among the
+ * localization evidence of Sec. 4 (the "latest-rank tie set"; Fig. 1 has a
+ * real tie at the backward boundary): ties[t,s] = #{r : P[t,r,s] = F[t,s]},
+ * the number of ranks whose prefix reaches the frontier.  1 marks a unique
+ * lead rank; more, a tie that sf_frontier resolved to the lowest rank.
+ *   d       [T][R][S] durations (device, 16-byte aligned).
+ *   a       [T][S] increments from sf_frontier on the same d (device, 8-byte
+ *           aligned); F[t,s] is rebuilt as their prefix over s.
+ *   ties    [T][S] int32 (device, 4-byte aligned, caller-owned).
+ *   status  device error word (nullable): SF_ST_NEGATIVE / SF_ST_RANGE as in
+ *           sf_frontier.
+ * Reads d once more (one CTA per step range).  Errors: SF_EINVAL (null d, a
+ * or ties, bad shape), SF_EINVAL_ALIGN.
+ */
+sf_status sf_frontier_ties(const int64_t* d, int64_t T, int64_t R, int64_t S, const int64_t* a, int32_t* ties,
+                           uint32_t* status, cudaStream_t stream);
+
+/*
  * sf_window_aggregate - Eq. 2 numerators and denominators plus per-(stage,
  * rank) credit, fused into the frontier pass.  Global step g = t0 + t belongs
  * to window floor(g / W); output row i is global window floor(t0 / W) + i,

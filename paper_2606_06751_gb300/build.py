@@ -17,7 +17,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libstagefrontier.so")
-SOURCES = ["sf_stream.cu", "sf_select.cu", "sf_rank.cu", "sf_group.cu", "sf_ingest.cu", "sf_api.cu", "sf_static.cu", "sf_pipeline.cu"]
+SOURCES = ["sf_stream.cu", "sf_select.cu", "sf_rank.cu", "sf_group.cu", "sf_ingest.cu", "sf_api.cu", "sf_static.cu", "sf_pipeline.cu", "sf_ties.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -135,6 +135,13 @@ sf_status sf_frontier(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t
   return cuda_status(launch_stream_pass(j, stream));
 }
 
+sf_status sf_frontier_ties(const int64_t* d, int64_t T, int64_t R, int64_t S, const int64_t* a, int32_t* ties,
+                           uint32_t* status, cudaStream_t stream) {
+  if (!d || !a || !ties || !shape_ok(T, R, S)) return SF_EINVAL;
+  if (!aligned(d, 16) || !aligned(a, 8) || !aligned(ties, 4) || !aligned(status, 4)) return SF_EINVAL_ALIGN;
+  return cuda_status(launch_frontier_ties(d, T, R, S, a, ties, status, stream));
+}
+
 sf_status sf_window_aggregate(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t t0, int64_t W,
                               int64_t* X, int64_t* D, int64_t* E, int32_t* C, uint8_t* step_lead,
                               int32_t accumulate, uint32_t* status, cudaStream_t stream) {

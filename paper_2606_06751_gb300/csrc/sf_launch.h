@@ -78,6 +78,9 @@ struct ZeroList {
 cudaError_t launch_zero_many(const ZeroList& z, cudaStream_t stream, bool* launched = nullptr);
 cudaError_t launch_wait_selftest(uint64_t limit_ns, uint32_t* status, cudaStream_t stream);
 cudaError_t launch_stream_pass(const StreamJob& job, cudaStream_t stream);
+// ties[t,s] = number of ranks whose prefix equals F[t,s] (F rebuilt from the increments a)
+cudaError_t launch_frontier_ties(const int64_t* d, int64_t T, int64_t R, int64_t S, const int64_t* a,
+                                 int32_t* ties, uint32_t* status, cudaStream_t stream);
 cudaError_t launch_window_median(const int64_t* d, int64_t T, int64_t R, int64_t S, int64_t W,
                                  int64_t* m, uint32_t* status, cudaStream_t stream);
 cudaError_t launch_rank_select(const int64_t* d, int64_t T, int64_t R, int64_t S, int of_prefix, int64_t t0,

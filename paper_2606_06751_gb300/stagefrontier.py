@@ -51,6 +51,7 @@ def _load():
     P, I, I32, S = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p
     sigs = {
         "sf_frontier": [P, I, I, I, P, P, P, P, S],
+        "sf_frontier_ties": [P, I, I, I, P, P, P, S],
         "sf_window_aggregate": [P, I, I, I, I, I, P, P, P, P, P, I32, P, S],
         "sf_topk_suspects": [P, P, I, I, I, I32, P, P, P, P, S],
         "sf_window_baselines": [P, I, I, I, I, I, P, P, P, P, I32, P, S],
@@ -182,6 +183,18 @@ def sf_frontier(d, a=None, lead=None, makespan=None, status=None, stream=None, o
     _check(_lib.sf_frontier(_p(d), T, R, S, _p(a), _p(lead), _p(makespan), _p(status), _stream(stream)),
            "sf_frontier")
     return Frontier(a, lead, makespan)
+
+
+def sf_frontier_ties(d, a=None, ties=None, status=None, stream=None):
+    """ties[t, s]: how many ranks reach the frontier F[t, s] (Sec. 4's tie set);
+    `a` are sf_frontier's increments on the same d (computed here when absent)."""
+    T, R, S = _d3(d)
+    if a is None:
+        a = sf_frontier(d, status=status, stream=stream, outputs=("a",)).a
+    ties = ties if ties is not None else _empty((T, S), torch.int32, d)
+    _check(_lib.sf_frontier_ties(_p(d), T, R, S, _p(a), _p(ties), _p(status), _stream(stream)),
+           "sf_frontier_ties")
+    return ties
 
 
 @dataclass

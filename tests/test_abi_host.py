@@ -55,6 +55,12 @@ FAKE = 1 << 20  # a well-aligned address that is never dereferenced: every call 
 
 def test_host_validation(sf):
     L = sf.lib()
+    # tie-set sizes: null d / a / ties, bad shape, misaligned d
+    assert L.sf_frontier_ties(None, 10, 4, 4, FAKE, FAKE, None, None) == sf.SF_EINVAL
+    assert L.sf_frontier_ties(FAKE, 10, 4, 4, None, FAKE, None, None) == sf.SF_EINVAL
+    assert L.sf_frontier_ties(FAKE, 10, 4, 4, FAKE, None, None, None) == sf.SF_EINVAL
+    assert L.sf_frontier_ties(FAKE, 0, 4, 4, FAKE, FAKE, None, None) == sf.SF_EINVAL
+    assert L.sf_frontier_ties(FAKE + 8, 10, 4, 4, FAKE, FAKE, None, None) == sf.SF_EINVAL_ALIGN
     # null input, bad shapes, no outputs
     assert L.sf_frontier(None, 10, 4, 4, FAKE, None, None, None, None) == sf.SF_EINVAL
     assert L.sf_frontier(FAKE, 0, 4, 4, FAKE, None, None, None, None) == sf.SF_EINVAL

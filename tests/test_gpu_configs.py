@@ -78,13 +78,16 @@ def test_sweep_frontier_full(sf, R, S):
     w = wl.sweep(R, S)
     d_np = w.generate()
     st = sf.new_status("cuda")
-    f = sf.sf_frontier(_to_dev(d_np), status=st)
+    d = _to_dev(d_np)
+    f = sf.sf_frontier(d, status=st)
+    ties = sf.sf_frontier_ties(d, a=f.a, status=st)
     torch.cuda.synchronize()
     assert int(st.item()) == 0
     o = O.frontier(d_np)
     assert np.array_equal(f.a.cpu().numpy(), o.a)
     assert np.array_equal(f.lead.cpu().numpy(), o.lead)
     assert np.array_equal(f.makespan.cpu().numpy(), o.makespan)
+    assert np.array_equal(ties.cpu().numpy(), o.ties)
 
 
 def test_streamed_chunks_match_resident(sf):

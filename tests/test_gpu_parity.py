@@ -92,6 +92,19 @@ def test_frontier_parity(sf, T, R, S, kind):
     assert np.array_equal(host(f.makespan), o.makespan)
 
 
+@pytest.mark.parametrize("T,R,S", SHAPES[:10] + SHAPES[14:] + LANES[:6] + GENERIC)
+@pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal"])
+def test_frontier_ties_parity(sf, T, R, S, kind):
+    """Size of the lead rank's tie set per step and stage against the oracle."""
+    d_np = make(T, R, S, T * 7 + R + S, kind)
+    o = O.frontier(d_np)
+    st = sf.new_status("cuda")
+    ties = sf.sf_frontier_ties(dev(d_np), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert np.array_equal(host(ties), o.ties)
+
+
 # Long step ranges: every CTA streams many tiles, so every ring stage is reused
 # many times (both regimes, both passes).
 LONG = [(200000, 8, 6), (20000, 64, 4), (8000, 128, 8), (3000, 512, 4), (1500, 1024, 10),
