@@ -44,6 +44,15 @@ def make(T, R, S, seed, kind):
     # lognormal around ms medians with one sync stage (realistic skew)
     med = rng.uniform(1e6, 5e7, size=S)
     x = np.rint(med * np.exp(0.1 * rng.standard_normal((T, R, S)))).astype(np.int64)
+    if kind == "mixed":     # wide rows among narrow ones (the kernels' 32-bit path takes only
+        # rows whose values stay below 2^(31 - ceil(log2 S))): one long stage in some rows, and
+        # copies of the rank below with a 2^32 ns last stage, equal prefixes across the two paths
+        t1, r1 = np.nonzero(rng.random((T, R)) < 0.05)
+        x[t1, r1, rng.integers(0, S, size=t1.size)] = rng.integers(1 << 26, 1 << 33, size=t1.size)
+        if R > 1:
+            t2, r2 = np.nonzero(rng.random((T, R - 1)) < 0.05)
+            x[t2, r2 + 1] = x[t2, r2]
+            x[t2, r2 + 1, S - 1] += 1 << 32
     return x
 
 
@@ -79,7 +88,7 @@ GENERIC = [(23, 9, 11), (10, 5, 14), (17, 33, 7), (12, 101, 4), (8, 30, 24), (30
 
 
 @pytest.mark.parametrize("T,R,S", SHAPES + GROUPED[4:] + LANES + GENERIC)
-@pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal"])
+@pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal", "mixed"])
 def test_frontier_parity(sf, T, R, S, kind):
     d_np = make(T, R, S, T * 131 + R * 7 + S, kind)
     o = O.frontier(d_np)
@@ -103,6 +112,31 @@ def test_frontier_ties_parity(sf, T, R, S, kind):
     torch.cuda.synchronize()
     assert int(st.item()) == 0
     assert np.array_equal(host(ties), o.ties)
+
+
+@pytest.mark.parametrize("T,R,S", [(40, 64, 4), (30, 128, 8), (200, 256, 4), (20, 512, 4), (300, 1000, 10),
+                                   (12, 1024, 10), (9, 4096, 2), (25, 48, 16), (7, 300, 6)])
+@pytest.mark.parametrize("wide_even", [True, False])
+def test_frontier_ties_across_narrow_and_wide_rows(sf, T, R, S, wide_even):
+    """Every rank has the same durations except a 2^32 ns last stage on every
+    other rank, so at every boundary before the last all ranks reach the
+    frontier together, half of them on the 32-bit path and half on the 64-bit
+    one: the lead rank must be rank 0 either way, and rank 0 or 1 at the last."""
+    rng = np.random.default_rng(T + R + S)
+    row = rng.integers(1, 1000, size=(T, 1, S), dtype=np.int64)
+    d_np = np.repeat(row, R, axis=1)
+    d_np[:, (0 if wide_even else 1)::2, S - 1] += 1 << 32
+    o = O.frontier(d_np)
+    st = sf.new_status("cuda")
+    f = sf.sf_frontier(dev(d_np), status=st)
+    g = sf.sf_window_aggregate(dev(d_np), 5, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert np.array_equal(host(f.a), o.a) and np.array_equal(host(f.lead), o.lead)
+    assert (o.lead[:, :S - 1] == 0).all()
+    ow = O.windows(d_np, 5)
+    for name in ("X", "D", "E", "C", "step_lead"):
+        assert np.array_equal(host(getattr(g, name)), getattr(ow, name)), name
 
 
 # Long step ranges: every CTA streams many tiles, so every ring stage is reused
