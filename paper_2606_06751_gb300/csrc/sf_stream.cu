@@ -6,7 +6,9 @@
 //     stage);
 //   * evidence pass (Sec. 4 Eq. 4): the same frontier plus, for every stage s,
 //     the makespan after replacing s by the clipped per-rank window median,
-//     per-step leader confidence and the telemetry-quality sums (App. A).
+//     per-step leader confidence and the telemetry-quality sums (App. A);
+//   * routing-baseline pass (Sec. 3 Props 1-2, Sec. 6): per-stage maxima and
+//     sums, the slowest rank and rank 0 per window.
 //
 // Fast path (S even, S <= 16, R*S a multiple of 16): a persistent grid, one
 // CTA per SM, each CTA owning a contiguous range of steps.  One producer
@@ -20,9 +22,15 @@
 // stages; larger steps by one warp group per step, spread over one or more
 // tiles, with two or four groups taking steps of one or two tiles in turn
 // (each group owning its ring stages) and all eight warps on larger steps.
+// The frontier over steps of up to 6 KB takes 2-8 steps per warp instruction
+// (lanes_kernel: groups of lanes, one step each).  Fewer steps than SMs over
+// many ranks split each step's ranks over a thread-block cluster
+// (split_frontier_kernel).
 //
 // Generic path (any other S <= 32 or R): one CTA per step range with plain
-// global loads.  Both paths share the per-step epilogues.
+// global loads.  All paths share the per-step epilogues.  A pass that follows
+// the clear of its own outputs starts as that clear's programmatic dependent
+// and writes only after griddep_wait().
 #include <algorithm>
 #include <array>
 #include <numeric>
