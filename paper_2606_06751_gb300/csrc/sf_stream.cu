@@ -1265,18 +1265,47 @@ cudaError_t dispatch_split(int S, const int64_t* d, const Params& p, int csize, 
 }
 
 // --------------------------------------------------------------------------
+// Untiled bulk copy global -> shared (both 16-byte aligned, a multiple of 16
+// bytes), completion counted in bytes on `bar`.
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
+
+// Orders this CTA's earlier shared-memory accesses (generic proxy) before
+// later bulk copies into shared memory (async proxy).
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // Generic path: any S <= 32, any R; one CTA of 256 threads per step range.
 // The per-stage state is sized by the bound SMAX >= S (4, 8, 16 or 32) and
 // every stage loop is unrolled to SMAX with an `s < S` guard, so the state
 // stays in registers.
 constexpr int kGenThreads = 256;
 
-template <int SMAX, int MODE, bool VEC>
+// RING: the CTA's steps are one contiguous byte range of d, streamed with
+// bulk copies in kGenRingStages chunks of p.stage_bytes (a power of two) into
+// a shared-memory ring; rows are read from the ring at their offset in that
+// range (a row may straddle chunks), and only a row past the range's last
+// 16-byte boundary is read from global memory.  Thread 0 refills the chunks
+// the finished step no longer needs right after the step's closing barrier,
+// so no stage is overwritten while a thread still reads it.  A step must fit
+// in kGenRingStages - 1 chunks (checked by the host).
+constexpr uint32_t kGenRingStages = 8;
+
+template <int SMAX, int MODE, bool VEC, bool RING>
 __global__ void __launch_bounds__(kGenThreads)
     stream_generic_kernel(const int64_t* __restrict__ d, const Params p) {
   constexpr bool GAIN = MODE == 1;
   constexpr bool BASE = MODE == 2;
+  constexpr uint32_t NST = kGenRingStages;
   __shared__ uint64_t red[kGenThreads / 32][66];
+  __shared__ uint64_t full[RING ? NST : 1];
+  __shared__ int abort_word;
+  extern __shared__ __align__(128) unsigned char ring[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int S = static_cast<int>(p.S);
   const int64_t R = p.R;
@@ -1287,10 +1316,50 @@ __global__ void __launch_bounds__(kGenThreads)
   QualAcc qa;
   WinTrack qt;  // window of the step a warp is on (evidence pass)
   BaseAcc bacc;
+  // ring geometry (RING only): bytes [A0, B0) of d, chunk c in stage c % NST
+  const int64_t RS8 = R * S * 8;
+  const uint32_t CB = static_cast<uint32_t>(p.stage_bytes);
+  const uint32_t cshift = RING ? static_cast<uint32_t>(__ffs(static_cast<int>(CB)) - 1) : 0u;
+  const uint32_t RBmask = NST * CB - 1;
+  const int64_t A0 = (t_begin * RS8) & ~int64_t(15), B0 = (t_end * RS8) & ~int64_t(15);
+  const int64_t nchunks = RING && B0 > A0 ? (B0 - A0 + CB - 1) >> cshift : 0;
+  const unsigned char* dbytes = reinterpret_cast<const unsigned char*>(d);
+  volatile int* abort = &abort_word;
+  int64_t issued = 0, released = 0;  // thread 0: chunks issued; chunks no step needs any more
+  auto issue = [&](int64_t c) {
+    const uint32_t st = static_cast<uint32_t>(c) & (NST - 1);
+    const int64_t off = A0 + (c << cshift);
+    const uint32_t bytes = static_cast<uint32_t>(min(int64_t(CB), B0 - off));
+    mbar_arrive_expect_tx(&full[st], bytes);
+    bulk_load(ring + size_t(st) * CB, dbytes + off, bytes, &full[st]);
+  };
+  if constexpr (RING) {
+    if (threadIdx.x == 0) {
+      for (uint32_t i = 0; i < NST; ++i) mbar_init(&full[i], 1);
+      *abort = 0;
+      fence_barrier_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0)
+      while (issued < nchunks && issued < int64_t(NST)) issue(issued++);
+  }
   griddep_wait();  // outputs cleared by the launch before this one (when it is its dependent)
   for (int64_t t = t_begin; t < t_end; ++t) {
     const int64_t w = GAIN ? qt.at(t, 0, p.W, 0) : 0;
     if (GAIN && p.quality) qual_window(p, qa, w, lane);
+    const int64_t s0 = t * RS8;  // the step's first byte
+    bool have = true;
+    if constexpr (RING) {
+      const int64_t s1 = min(s0 + RS8, B0);
+      if (s1 > s0)
+        for (int64_t c = (s0 - A0) >> cshift; c <= (s1 - 1 - A0) >> cshift; ++c)
+          have &= mbar_wait_bounded(&full[static_cast<uint32_t>(c) & (NST - 1)],
+                                    static_cast<uint32_t>(c >> ceil_log2(NST)) & 1u, abort);
+    }
+    // one rank row's durations: from the ring when the whole row lies below
+    // B0 (ring offsets wrap), else from global memory
+    auto in_ring = [&](int64_t r) { return RING && s0 + (r + 1) * S * 8 <= B0; };
+    auto ring_off = [&](int64_t r) { return static_cast<uint32_t>(s0 + r * S * 8 - A0) & RBmask; };
     int64_t b0[SMAX], b1[SMAX];
     int32_t br[SMAX];
     uint64_t slow = 0;
@@ -1305,11 +1374,17 @@ __global__ void __launch_bounds__(kGenThreads)
       // '>' keeps the lowest rank), each duration loaded where it is used
       for (int64_t r = threadIdx.x; r < R; r += kGenThreads) {
         const int64_t* row = d + (t * R + r) * S;
+        const bool rr = in_ring(r);
+        const uint32_t ro = RING ? ring_off(r) : 0u;
+        auto val = [&](int s) -> int64_t {
+          if (RING && rr) return *reinterpret_cast<const int64_t*>(ring + ((ro + 8u * s) & RBmask));
+          return __ldg(row + s);
+        };
         int64_t P = 0, other = 0;
 #pragma unroll
         for (int s = 0; s < SMAX; ++s) {
           if (s >= S) break;
-          const int64_t v = __ldg(row + s);
+          const int64_t v = have ? val(s) : 0;
           dor |= hi32(v);
           P += v;
           if (s == p.other_stage) other = v;
@@ -1331,7 +1406,7 @@ __global__ void __launch_bounds__(kGenThreads)
 #pragma unroll
           for (int s = 0; s < SMAX; ++s) {
             if (s >= S) break;
-            int64_t cut = __ldg(row + s) - __ldg(mr + s);
+            int64_t cut = (have ? val(s) : 0) - __ldg(mr + s);
             cut = cut > 0 ? cut : 0;
             b1[s] = (P - cut) > b1[s] ? (P - cut) : b1[s];
           }
@@ -1344,11 +1419,18 @@ __global__ void __launch_bounds__(kGenThreads)
       static_assert(!GAIN, "the evidence pass loads durations where it uses them");
       for (int64_t r = threadIdx.x; r < R; r += kGenThreads) {
         const int64_t* row = d + (t * R + r) * S;
+        const bool rr = in_ring(r);
+        const uint32_t ro = RING ? ring_off(r) : 0u;
         int64_t v[SMAX];
 #pragma unroll
         for (int s = 0; s < SMAX; s += 2) {
           if (s >= S) break;
-          const longlong2 x = __ldg(reinterpret_cast<const longlong2*>(row + s));
+          longlong2 x = make_longlong2(0, 0);
+          if (RING && rr) {
+            if (have) x = *reinterpret_cast<const longlong2*>(ring + ((ro + 8u * s) & RBmask));
+          } else {
+            x = __ldg(reinterpret_cast<const longlong2*>(row + s));
+          }
           v[s] = x.x;
           v[s + 1] = x.y;
         }
@@ -1408,11 +1490,29 @@ __global__ void __launch_bounds__(kGenThreads)
       else finalize_frontier(p, S, t, v0, lane, acc);
     }
     __syncthreads();
+    if constexpr (RING) {
+      // every thread is done with step t: the chunks wholly before the next
+      // step's first byte are free, and each freed stage takes the next chunk
+      if (threadIdx.x == 0) {
+        const int64_t free_upto = min(nchunks, (s0 + RS8 - A0) >> cshift);
+        if (released < free_upto && issued < nchunks) fence_proxy_async_smem();
+        for (; released < free_upto; ++released)
+          if (issued < nchunks) issue(issued++);
+      }
+    }
+  }
+  if constexpr (RING) {
+    // copies still in flight (only when a wait gave up): let them land before
+    // the CTA's shared memory is released
+    if (threadIdx.x == 0)
+      for (int64_t c = released; c < issued; ++c)
+        mbar_wait_timeout(&full[static_cast<uint32_t>(c) & (NST - 1)], static_cast<uint32_t>(c >> ceil_log2(NST)) & 1u);
   }
   if (BASE && warp == 0) flush_base(p, S, bacc, lane);
   if (!BASE && p.X && warp == 0) flush_window(p, S, acc, lane);
   if (GAIN && p.quality) qual_window(p, qa, -2, lane);
-  const uint32_t bits = range_bits(__reduce_or_sync(kFull, dor), __reduce_or_sync(kFull, tor));
+  const uint32_t bits = range_bits(__reduce_or_sync(kFull, dor), __reduce_or_sync(kFull, tor)) |
+                        ((RING && *abort) ? SF_ST_TIMEOUT : 0u);
   if (lane == 0) report(p.status, bits);
 }
 
@@ -1620,17 +1720,51 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
     return j.gain ? dispatch_fast<1>(static_cast<int>(j.S), map, map_m, p, grid, stream, pdl)
                   : dispatch_fast<0>(static_cast<int>(j.S), map, map_m, p, grid, stream, pdl);
   }
-  const int grid = static_cast<int>(std::min<int64_t>(int64_t(sms) * 4, j.T));
   count_launch();
   const bool vec = j.S % 2 == 0;  // whole-row 16-byte loads (frontier and baseline passes)
+  // bulk-copy ring: the smallest power-of-two chunk (4-16 KB) of which
+  // kGenRingStages - 1 hold a whole step; larger steps read global memory
+  const int64_t step_bytes = j.R * j.S * 8;
+  uint32_t chunk = 0;
+  for (uint32_t c = 4096; c <= 16384 && !chunk; c *= 2)
+    if (step_bytes <= int64_t(kGenRingStages - 1) * c) chunk = c;
+  p.stage_bytes = static_cast<int>(chunk);
+  p.nst = static_cast<int>(kGenRingStages);
   auto generic = [&](auto smax) {
     constexpr int SM = decltype(smax)::value;
     const bool pdl = j.after_clear;
-    if (j.gain) return launch_ex(stream_generic_kernel<SM, 1, false>, grid, kGenThreads, 0, stream, pdl, j.d, p);
-    if (j.base && vec) return launch_ex(stream_generic_kernel<SM, 2, true>, grid, kGenThreads, 0, stream, pdl, j.d, p);
-    if (j.base) return launch_ex(stream_generic_kernel<SM, 2, false>, grid, kGenThreads, 0, stream, pdl, j.d, p);
-    if (vec) return launch_ex(stream_generic_kernel<SM, 0, true>, grid, kGenThreads, 0, stream, pdl, j.d, p);
-    return launch_ex(stream_generic_kernel<SM, 0, false>, grid, kGenThreads, 0, stream, pdl, j.d, p);
+    auto go = [&](auto kern, bool ring) {
+      const size_t smem = ring ? size_t(kGenRingStages) * chunk : 0;
+      int per_sm = 4;
+      if (ring) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             static_cast<int>(smem));
+        if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kGenThreads, smem);
+        if (e != cudaSuccess) return e;
+        per_sm = std::max(per_sm, 1);
+      }
+      const int grid = static_cast<int>(std::min<int64_t>(int64_t(sms) * per_sm, j.T));
+      return launch_ex(kern, grid, kGenThreads, smem, stream, pdl, j.d, p);
+    };
+    if constexpr (SM > 16) {
+      // more than 16 stages: registers hold these kernels to one or two CTAs
+      // per SM, and the bulk-copy ring keeps the loads off their step chain
+      // (512 x 24: 0.434 -> 0.405 ms).  Up to 16 stages four CTAs per SM
+      // hide the loads better than a ring that leaves room for three (1000 x 5:
+      // 0.229 against 0.285 ms), so those shapes read global memory.
+      if (chunk != 0) {
+        if (j.gain) return go(stream_generic_kernel<SM, 1, false, true>, true);
+        if (j.base && vec) return go(stream_generic_kernel<SM, 2, true, true>, true);
+        if (j.base) return go(stream_generic_kernel<SM, 2, false, true>, true);
+        if (vec) return go(stream_generic_kernel<SM, 0, true, true>, true);
+        return go(stream_generic_kernel<SM, 0, false, true>, true);
+      }
+    }
+    if (j.gain) return go(stream_generic_kernel<SM, 1, false, false>, false);
+    if (j.base && vec) return go(stream_generic_kernel<SM, 2, true, false>, false);
+    if (j.base) return go(stream_generic_kernel<SM, 2, false, false>, false);
+    if (vec) return go(stream_generic_kernel<SM, 0, true, false>, false);
+    return go(stream_generic_kernel<SM, 0, false, false>, false);
   };
   if (j.S <= 4) return generic(std::integral_constant<int, 4>{});
   if (j.S <= 8) return generic(std::integral_constant<int, 8>{});
