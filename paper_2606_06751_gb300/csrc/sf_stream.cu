@@ -1516,6 +1516,149 @@ __global__ void __launch_bounds__(kGenThreads)
   if (lane == 0) report(p.status, bits);
 }
 
+// Warp-per-step generic path (S <= 16, many steps): each warp takes every
+// eighth step of its CTA's range alone (rank rows lane, lane + 32, ... in
+// increasing order, so a strict '>' keeps the lowest rank), reduces the
+// stages with warp reductions and runs the step's epilogue itself, with its
+// own window accumulators: no CTA barrier, eight independent steps in flight
+// per CTA.  (The CTA-per-step kernel above spends about 5 us per step behind
+// two barriers.)
+template <int SMAX, int MODE, bool VEC>
+__global__ void __launch_bounds__(kGenThreads)
+    stream_warp_kernel(const int64_t* __restrict__ d, const Params p) {
+  constexpr bool GAIN = MODE == 1;
+  constexpr bool BASE = MODE == 2;
+  constexpr int UG = SMAX > 8 ? 1 : 2;  // rank rows in flight per lane (frontier, baselines)
+  constexpr int kWarps = kGenThreads / 32;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int S = static_cast<int>(p.S);
+  const int64_t R = p.R;
+  const int64_t NB = gridDim.x, b = blockIdx.x;
+  const int64_t t_begin = p.T * b / NB, t_end = p.T * (b + 1) / NB;
+  uint32_t dor = 0, tor = 0;
+  WinAcc acc;
+  QualAcc qa;
+  WinTrack qt;  // window of the warp's step (evidence pass)
+  BaseAcc bacc;
+  griddep_wait();  // outputs cleared by the launch before this one (when it is its dependent)
+  for (int64_t t = t_begin + warp; t < t_end; t += kWarps) {
+    const int64_t w = GAIN ? qt.at(t, 0, p.W, 0) : 0;
+    if (GAIN && p.quality) qual_window(p, qa, w, lane);
+    int64_t b0[SMAX], b1[SMAX];
+    int32_t br[SMAX];
+    uint64_t slow = 0;
+#pragma unroll
+    for (int s = 0; s < SMAX; ++s) {
+      b0[s] = BASE ? 0 : -1;
+      b1[s] = 0;
+      br[s] = 0;
+    }
+    if constexpr (GAIN) {
+      // evidence pass: one row at a time, durations loaded where used
+      for (int64_t r = lane; r < R; r += 32) {
+        const int64_t* row = d + (t * R + r) * S;
+        int64_t P = 0, other = 0;
+#pragma unroll
+        for (int s = 0; s < SMAX; ++s) {
+          if (s >= S) break;
+          const int64_t v = __ldg(row + s);
+          dor |= hi32(v);
+          P += v;
+          if (s == p.other_stage) other = v;
+          if (P > b0[s]) {
+            b0[s] = P;
+            br[s] = static_cast<int32_t>(r);
+          }
+        }
+        tor |= hi32(P);
+        const int64_t* mr = p.m + (w * R + r) * S;
+#pragma unroll
+        for (int s = 0; s < SMAX; ++s) {
+          if (s >= S) break;
+          int64_t cut = __ldg(row + s) - __ldg(mr + s);
+          cut = cut > 0 ? cut : 0;
+          b1[s] = (P - cut) > b1[s] ? (P - cut) : b1[s];
+        }
+        if (p.quality) qual_row(p, qa, t, r, P, other, dor);
+      }
+    } else {
+      for (int64_t r0 = lane; r0 < R; r0 += 32 * UG) {
+        int64_t v[UG][SMAX];
+#pragma unroll
+        for (int u = 0; u < UG; ++u) {
+          const int64_t r = r0 + 32 * u;
+          if (r >= R) break;
+          const int64_t* row = d + (t * R + r) * S;
+          if constexpr (VEC) {  // S even: rows start 16-byte aligned
+#pragma unroll
+            for (int s = 0; s < SMAX; s += 2) {
+              if (s >= S) break;
+              const longlong2 x = __ldg(reinterpret_cast<const longlong2*>(row + s));
+              v[u][s] = x.x;
+              v[u][s + 1] = x.y;
+            }
+          } else {
+#pragma unroll
+            for (int s = 0; s < SMAX; ++s) {
+              if (s >= S) break;
+              v[u][s] = __ldg(row + s);
+            }
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < UG; ++u) {
+          const int64_t r = r0 + 32 * u;
+          if (r >= R) break;
+          int64_t P = 0;
+#pragma unroll
+          for (int s = 0; s < SMAX; ++s) {
+            if (s >= S) break;
+            dor |= hi32(v[u][s]);
+            P += v[u][s];
+            if (BASE) {
+              b0[s] = v[u][s] > b0[s] ? v[u][s] : b0[s];
+              b1[s] += v[u][s];
+            } else if (P > b0[s]) {
+              b0[s] = P;
+              br[s] = static_cast<int32_t>(r);
+            }
+          }
+          tor |= hi32(P);
+          if (BASE) {
+            const uint64_t k = (static_cast<uint64_t>(P) << 16) | static_cast<uint64_t>(65535 - r);
+            slow = k > slow ? k : slow;
+          }
+        }
+      }
+    }
+    // lane s keeps stage s's reductions
+    uint64_t v0 = 0, v1 = 0;
+#pragma unroll
+    for (int s = 0; s < SMAX; ++s) {
+      if (s >= S) break;
+      uint64_t k0;
+      if (BASE) k0 = static_cast<uint64_t>(b0[s]);
+      else k0 = b0[s] < 0 ? 0ull : (static_cast<uint64_t>(b0[s]) << 16) | static_cast<uint64_t>(65535 - br[s]);
+      const uint64_t m0 = warp_max_u64(k0);
+      const uint64_t m1 = GAIN   ? warp_max_u64(static_cast<uint64_t>(b1[s]))
+                          : BASE ? warp_sum_u64(static_cast<uint64_t>(b1[s]))
+                                 : 0;
+      if (lane == s) {
+        v0 = m0;
+        v1 = m1;
+      }
+    }
+    if (GAIN) finalize_gain(p, S, t, v0, static_cast<int64_t>(v1), lane, acc);
+    else if (BASE) finalize_base(p, S, t, v0, v1, warp_max_u64(slow), lane, bacc);
+    else finalize_frontier(p, S, t, v0, lane, acc);
+  }
+  if (BASE) flush_base(p, S, bacc, lane);
+  if (!BASE && p.X) flush_window(p, S, acc, lane);
+  if (GAIN && p.quality) qual_window(p, qa, -2, lane);
+  const uint32_t bits = range_bits(__reduce_or_sync(kFull, dor), __reduce_or_sync(kFull, tor));
+  if (lane == 0) report(p.status, bits);
+}
+
 // --------------------------------------------------------------------------
 // Host side
 
@@ -1758,6 +1901,25 @@ cudaError_t launch_stream_pass(const StreamJob& j, cudaStream_t stream) {
         if (j.base) return go(stream_generic_kernel<SM, 2, false, true>, true);
         if (vec) return go(stream_generic_kernel<SM, 0, true, true>, true);
         return go(stream_generic_kernel<SM, 0, false, true>, true);
+      }
+    }
+    if constexpr (SM <= 16) {
+      // many steps: one warp per step (see stream_warp_kernel); few steps
+      // keep a CTA per step so that a step's ranks still spread over 256 threads
+      if (j.T >= int64_t(sms) * 4 * (kGenThreads / 32)) {
+        auto gow = [&](auto kern) {
+          int per_sm = 1;
+          cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kGenThreads, 0);
+          if (e != cudaSuccess) return e;
+          const int grid = static_cast<int>(std::min<int64_t>(int64_t(sms) * std::max(per_sm, 1),
+                                                              (j.T + kGenThreads / 32 - 1) / (kGenThreads / 32)));
+          return launch_ex(kern, grid, kGenThreads, 0, stream, pdl, j.d, p);
+        };
+        if (j.gain) return gow(stream_warp_kernel<SM, 1, false>);
+        if (j.base && vec) return gow(stream_warp_kernel<SM, 2, true>);
+        if (j.base) return gow(stream_warp_kernel<SM, 2, false>);
+        if (vec) return gow(stream_warp_kernel<SM, 0, true>);
+        return gow(stream_warp_kernel<SM, 0, false>);
       }
     }
     if (j.gain) return go(stream_generic_kernel<SM, 1, false, false>, false);

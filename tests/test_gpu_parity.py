@@ -85,9 +85,11 @@ LANES = [(257, 376, 2), (300, 104, 2), (999, 40, 2), (211, 184, 4), (405, 52, 4)
 # multiple of 16, more than 16 stages): every stage bound of its kernels
 # (S <= 4, <= 8, <= 16, <= 32)
 GENERIC = [(23, 9, 11), (10, 5, 14), (17, 33, 7), (12, 101, 4), (8, 30, 24), (300, 1000, 5)]
+# generic shapes with many steps (at least 4 x 8 per SM): one warp per step
+GENERIC_MANY = [(6000, 9, 11), (6000, 33, 7), (6000, 10, 3), (6000, 5, 14), (6000, 7, 6)]
 
 
-@pytest.mark.parametrize("T,R,S", SHAPES + GROUPED[4:] + LANES + GENERIC)
+@pytest.mark.parametrize("T,R,S", SHAPES + GROUPED[4:] + LANES + GENERIC + GENERIC_MANY)
 @pytest.mark.parametrize("kind", ["ties", "zeros", "lognormal", "mixed"])
 def test_frontier_parity(sf, T, R, S, kind):
     d_np = make(T, R, S, T * 131 + R * 7 + S, kind)
@@ -172,7 +174,8 @@ def test_long_ranges_reuse_ring(sf, T, R, S):
     assert np.array_equal(host(ev.Y)[:2], O.direct_gain(d_np[:2 * W], W, m2))
 
 
-@pytest.mark.parametrize("T,R,S", SHAPES[:4] + SHAPES[5:9] + SHAPES[14:18] + GROUPED + LANES + GENERIC)
+@pytest.mark.parametrize("T,R,S", SHAPES[:4] + SHAPES[5:9] + SHAPES[14:18] + GROUPED + LANES + GENERIC
+                         + GENERIC_MANY)
 @pytest.mark.parametrize("t0,W", [(0, 7), (13, 10), (0, 1000)])
 def test_window_aggregate_parity(sf, T, R, S, t0, W):
     d_np = make(T, R, S, T + R + S + t0, "ties" if R < 100 else "lognormal")
@@ -268,7 +271,8 @@ def test_median_parity(sf, T, R, S, W, kind):
 @pytest.mark.parametrize("T,R,S,W", [(120, 8, 6, 50), (64, 128, 8, 30), (40, 1024, 10, 16),
                                      (33, 3, 5, 10), (20, 8192, 8, 8), (30, 64, 16, 30), (9, 5, 4, 1),
                                      (11, 40, 8, 2), (23, 9, 11, 5), (17, 33, 7, 4), (8, 30, 24, 3),
-                                     (12, 101, 4, 6), (10, 5, 14, 3)])
+                                     (12, 101, 4, 6), (10, 5, 14, 3), (6000, 9, 11, 100), (6000, 33, 7, 250),
+                                     (6000, 10, 3, 1000), (6000, 5, 14, 64)])
 def test_direct_gain_parity(sf, T, R, S, W):
     d_np = make(T, R, S, R + S, "lognormal")
     m_np = O.window_median(d_np, W)
@@ -397,7 +401,8 @@ def test_bounded_wait_times_out_cleanly(sf):
     assert np.array_equal(host(f.a), O.frontier(host(d)).a)
 
 
-@pytest.mark.parametrize("T,R,S", SHAPES[:4] + SHAPES[5:9] + SHAPES[14:18] + GROUPED + GENERIC + [(200000, 8, 6)])
+@pytest.mark.parametrize("T,R,S", SHAPES[:4] + SHAPES[5:9] + SHAPES[14:18] + GROUPED + GENERIC + GENERIC_MANY
+                         + [(200000, 8, 6)])
 @pytest.mark.parametrize("t0,W", [(0, 7), (13, 100)])
 def test_baselines_parity(sf, T, R, S, t0, W):
     """Per-stage max, sum (128-bit), slowest-rank breakdown and rank-0 total
