@@ -28,8 +28,9 @@
  *   - Valid durations satisfy 0 <= d < 2^47 and every rank total
  *     P[t,r,S-1] < 2^47 ns (about 39 hours per step); anything else sets
  *     SF_ST_NEGATIVE or SF_ST_RANGE.  All sums over a window then fit int64.
- *   - Ties: the lead rank of (t,s) is the LOWEST rank attaining F[t,s]; the
- *     leading stage of a step is the lowest stage with the largest increment.
+ *   - Ties: the lead rank of (t,s) is the LOWEST rank attaining F[t,s] (how
+ *     many ranks attain it is reported by sf_frontier_ties); the leading stage
+ *     of a step is the lowest stage with the largest increment.
  *   - Integer outputs are exact and deterministic (integer atomics commute);
  *     fp64 outputs are one IEEE division of two int64 values.
  */
